@@ -1,0 +1,247 @@
+"""Pins of the fp64 oracle to facts fixed by the paper and by mathematics.
+
+Each ``pin_*`` function runs one check against an oracle build (``lib=None``
+is the real oracle) and raises AssertionError when the oracle disagrees.
+They are collected by test_oracle_pins.py (the real oracle must pass all of
+them) and test_oracle_mutants.py (every deliberately broken build must fail at
+least one of them).
+
+What pins what:
+  * Eq. 1 + causal mask      -> torch float64 scaled_dot_product_attention
+                                (gamma = 1, and window >= N where A* = A).
+  * sink + window set W(i)   -> closed-form counts |W(i)| and mean key index
+                                under uniform scores (Q = 0).
+  * Eq. 6 / Alg. 1 Delta     -> closed forms with K = 0 (prefix / window means),
+                                window = 1 (S_i = v_i), constant V, and the
+                                sampled-row identity A^V_{k gamma} = ~AV_k.
+  * GQA head mapping         -> explicit repetition of the KV heads.
+  * Lemma 1                  -> the appendix inequality on every sample.
+  * whole-matrix restatement -> the numpy brute force (oracle/brute.py).
+"""
+import numpy as np
+import torch
+
+import oracle
+from oracle import brute
+
+TOL = 1e-12
+
+
+def rand_bits(seed, shape, scale=1.0):
+    g = torch.Generator().manual_seed(seed)
+    x = (torch.randn(shape, generator=g, dtype=torch.float32) * scale).to(torch.bfloat16)
+    return x.view(torch.int16).numpy().view(np.uint16)
+
+
+def const_bits(shape, value):
+    x = torch.full(shape, value, dtype=torch.float32).to(torch.bfloat16)
+    return x.view(torch.int16).numpy().view(np.uint16)
+
+
+def f64(bits):
+    return oracle.bf16_bits_to_f64(bits)
+
+
+def _sdpa_causal(Qb, Kb, Vb):
+    Q, K, V = (torch.from_numpy(f64(x)) for x in (Qb, Kb, Vb))
+    G = Q.shape[1] // K.shape[1]
+    K = K.repeat_interleave(G, dim=1)
+    V = V.repeat_interleave(G, dim=1)
+    return torch.nn.functional.scaled_dot_product_attention(Q, K, V, is_causal=True).numpy()
+
+
+def _w_count(i, n_sink, window):
+    """Closed form |W(i)|: the band of min(i+1, window) keys ending at i plus
+    the sinks that lie before the band."""
+    band_start = max(0, i - window + 1)
+    return min(i + 1, window) + min(n_sink, band_start)
+
+
+def _w_index_sum(i, n_sink, window):
+    """Closed form sum of the key indices in W(i) (arithmetic series)."""
+    a = max(0, i - window + 1)
+    band = (a + i) * (i - a + 1) // 2
+    s = min(n_sink, a)
+    return band + s * (s - 1) // 2
+
+
+# --------------------------------------------------------------------------
+def pin_gamma1_is_sdpa(lib=None):
+    """gamma = 1: every row is sampled, Eq. 6 gives dense causal attention."""
+    for (B, Hq, Hkv, N, d, s, w) in [(1, 2, 2, 45, 16, 2, 7), (2, 4, 2, 33, 8, 0, 3)]:
+        Q, K, V = rand_bits(1, (B, Hq, N, d)), rand_bits(2, (B, Hkv, N, d)), rand_bits(3, (B, Hkv, N, d))
+        A = oracle.delta_attn(Q, K, V, s, w, 1, lib=lib)["A"]
+        ref = _sdpa_causal(Q, K, V)
+        assert np.abs(A - ref).max() <= TOL, "gamma=1 must equal dense causal attention"
+
+
+def pin_full_window_is_sdpa(lib=None):
+    """window >= N: W(i) = C(i), so A* = A and the output is dense attention."""
+    B, Hq, Hkv, N, d = 1, 4, 2, 40, 16
+    Q, K, V = rand_bits(4, (B, Hq, N, d), 2.0), rand_bits(5, (B, Hkv, N, d), 2.0), rand_bits(6, (B, Hkv, N, d))
+    for s, w, gamma in [(0, N, 8), (3, N + 5, 5), (1, N, 64)]:
+        out = oracle.delta_attn(Q, K, V, s, w, gamma, lib=lib)
+        ref = _sdpa_causal(Q, K, V)
+        assert np.abs(out["A"] - ref).max() <= TOL
+        assert np.abs(out["S"] - ref).max() <= TOL, "A*V must be dense when window >= N"
+
+
+def pin_zero_keys_closed_form(lib=None):
+    """K = 0: every score is 0, softmax is uniform over the key set, so
+    D_i = mean_{j<=i} v_j and S_i = mean_{j in W(i)} v_j (no exponentials)."""
+    B, Hq, Hkv, N, d = 1, 2, 1, 50, 8
+    Q = rand_bits(7, (B, Hq, N, d))
+    K = np.zeros((B, Hkv, N, d), np.uint16)
+    V = rand_bits(8, (B, Hkv, N, d))
+    Vf = f64(V)[0, 0]
+    pre = np.concatenate([np.zeros((1, d)), np.cumsum(Vf, axis=0)])
+    for s, w, gamma in [(2, 6, 4), (0, 1, 3), (5, 13, 7), (1, 3, 16)]:
+        out = oracle.delta_attn(Q, K, V, s, w, gamma, lib=lib)
+        for h in range(Hq):
+            for i in range(N):
+                a = max(0, i - w + 1)
+                cnt = (i - a + 1) + min(s, a)
+                S_i = (pre[i + 1] - pre[a] + pre[min(s, a)]) / cnt
+                assert np.abs(out["S"][0, h, i] - S_i).max() <= TOL
+                ks = (i // gamma) * gamma
+                aks = max(0, ks - w + 1)
+                S_k = (pre[ks + 1] - pre[aks] + pre[min(s, aks)]) / ((ks - aks + 1) + min(s, aks))
+                D_k = pre[ks + 1] / (ks + 1)
+                assert np.abs(out["A"][0, h, i] - (S_i + D_k - S_k)).max() <= TOL
+
+
+def pin_window1_no_sink(lib=None):
+    """window = 1, n_sink = 0: S_i = v_i, so A^V_i = v_i + D_{k gamma} - v_{k gamma}."""
+    B, Hq, Hkv, N, d = 1, 2, 2, 37, 16
+    Q, K, V = rand_bits(9, (B, Hq, N, d)), rand_bits(10, (B, Hkv, N, d)), rand_bits(11, (B, Hkv, N, d))
+    gamma = 6
+    out = oracle.delta_attn(Q, K, V, 0, 1, gamma, lib=lib)
+    dense = _sdpa_causal(Q, K, V)
+    Vf = f64(V)
+    for h in range(Hq):
+        assert np.abs(out["S"][0, h] - Vf[0, h]).max() <= TOL
+        for i in range(N):
+            ks = (i // gamma) * gamma
+            want = Vf[0, h, i] + dense[0, h, ks] - Vf[0, h, ks]
+            assert np.abs(out["A"][0, h, i] - want).max() <= TOL
+
+
+def pin_constant_values(lib=None):
+    """v_j = c for all j: every softmax average is c, Delta = 0."""
+    B, Hq, Hkv, N, d = 1, 2, 2, 30, 8
+    Q, K = rand_bits(12, (B, Hq, N, d), 3.0), rand_bits(13, (B, Hkv, N, d), 3.0)
+    V = const_bits((B, Hkv, N, d), 0.375)
+    out = oracle.delta_attn(Q, K, V, 2, 5, 4, lib=lib)
+    assert np.abs(out["A"] - 0.375).max() <= TOL
+
+
+def pin_mask_structure(lib=None):
+    """Q = 0 gives uniform weights over the key set.  With v_j[0] = 1,
+    v_j[1] = [j < n_sink], v_j[2] = j / 64 the sparse output exposes the set:
+    S_i[1] = (#sinks in W(i)) / |W(i)|, S_i[2] = mean index / 64."""
+    N, d = 64, 8
+    Q = np.zeros((1, 1, N, d), np.uint16)
+    K = rand_bits(14, (1, 1, N, d))
+    for s, w in [(4, 8), (0, 5), (3, 1), (10, 6), (2, 64)]:
+        Vf = np.zeros((1, 1, N, d), np.float32)
+        Vf[0, 0, :, 0] = 1.0
+        Vf[0, 0, :, 1] = (np.arange(N) < s)
+        Vf[0, 0, :, 2] = np.arange(N) / 64.0
+        V = torch.from_numpy(Vf).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+        out = oracle.delta_attn(Q, K, V, s, w, 4, lib=lib)
+        for i in range(N):
+            cnt = _w_count(i, s, w)
+            sinks_in = min(s, i + 1)
+            S = out["S"][0, 0, i]
+            assert abs(S[0] - 1.0) <= TOL
+            assert abs(S[1] - sinks_in / cnt) <= TOL, (i, s, w)
+            assert abs(S[2] - _w_index_sum(i, s, w) / 64.0 / cnt) <= TOL, (i, s, w)
+
+
+def pin_sampled_rows_are_dense(lib=None):
+    """Eq. 6 at i = k gamma: A^V = A*V + ~AV - A*V = the dense row; and row 0
+    attends to itself only, so A^V_0 = v_0."""
+    B, Hq, Hkv, N, d = 1, 4, 2, 53, 16
+    Q, K, V = rand_bits(15, (B, Hq, N, d)), rand_bits(16, (B, Hkv, N, d)), rand_bits(17, (B, Hkv, N, d))
+    gamma = 8
+    out = oracle.delta_attn(Q, K, V, 2, 9, gamma, lib=lib)
+    dense = _sdpa_causal(Q, K, V)
+    assert np.abs(out["A"][:, :, ::gamma] - dense[:, :, ::gamma]).max() <= TOL
+    Vf = f64(V)
+    for h in range(Hq):
+        assert np.abs(out["A"][0, h, 0] - Vf[0, h // 2, 0]).max() <= TOL
+    assert out["max_dev"] <= TOL, "softmax rows must sum to 1"
+
+
+def pin_gqa_repeat(lib=None):
+    """GQA: Hkv = 2 with Hq = 4 equals Hkv = 4 with each KV head repeated."""
+    B, Hq, Hkv, N, d = 2, 4, 2, 41, 16
+    Q, K, V = rand_bits(18, (B, Hq, N, d)), rand_bits(19, (B, Hkv, N, d)), rand_bits(20, (B, Hkv, N, d))
+    a = oracle.delta_attn(Q, K, V, 3, 7, 5, lib=lib)["A"]
+    Kr = np.ascontiguousarray(np.repeat(K, 2, axis=1))
+    Vr = np.ascontiguousarray(np.repeat(V, 2, axis=1))
+    b = oracle.delta_attn(Q, Kr, Vr, 3, 7, 5, lib=lib)["A"]
+    assert np.abs(a - b).max() <= TOL
+
+
+def pin_lemma1(lib=None):
+    """Appendix, Lemma 1: |Delta - sum_{omitted} a_j v_j| <= H/(H+T) max_W |v_j|,
+    on every sample of a problem with scaled sinks."""
+    B, Hq, Hkv, N, d = 1, 2, 1, 96, 16
+    Q, K, V = rand_bits(21, (B, Hq, N, d), 1.5), rand_bits(22, (B, Hkv, N, d), 1.5), rand_bits(23, (B, Hkv, N, d))
+    nontrivial = 0
+    for h in range(Hq):
+        for k in range(0, N // 8):
+            lhs, rhs, frac = oracle.lemma1(Q, K, V, 2, 16, 8, 0, h, k, lib=lib)
+            assert np.all(lhs <= rhs * (1 + 1e-9) + TOL), (h, k)
+            nontrivial += frac > 0.05
+    assert nontrivial > 0
+
+
+def pin_brute_force(lib=None):
+    """The direct per-row evaluation equals the whole-matrix restatement of
+    Alg. 1 (numpy) on small problems, over a sweep of gamma, window, sinks,
+    GQA ratio, both output modes and the dense tail."""
+    cases = []
+    for gamma in (1, 2, 3, 5, 16, 64):
+        for window in (1, 2, 7, 64):
+            for n_sink in (0, 1, 4):
+                cases.append((gamma, window, n_sink))
+    seed = 100
+    for idx, (gamma, window, n_sink) in enumerate(cases):
+        G = (1, 2, 4)[idx % 3]
+        Hkv = 1 + (idx % 2)
+        Hq = Hkv * G
+        N = (64, 37, 50)[idx % 3]
+        d = 8
+        seed += 1
+        Q, K, V = rand_bits(seed, (1, Hq, N, d), 1.5), rand_bits(seed + 1000, (1, Hkv, N, d), 1.5), \
+            rand_bits(seed + 2000, (1, Hkv, N, d))
+        mode = "recompute" if idx % 7 == 3 else "delta"
+        tail = 5 if idx % 11 == 4 else 0
+        A_b, S_b, _ = brute.delta_attn(f64(Q), f64(K), f64(V), n_sink, window, gamma, mode=mode, tail_dense=tail)
+        out = oracle.delta_attn(Q, K, V, n_sink, window, gamma, mode=mode, tail_dense=tail, lib=lib)
+        assert np.abs(out["A"] - A_b).max() <= TOL, (gamma, window, n_sink, mode, tail)
+        assert np.abs(out["S"] - S_b).max() <= TOL
+
+
+def pin_rows_agree(lib=None):
+    """oracle_rows (per-row) agrees with the box evaluation."""
+    B, Hq, Hkv, N, d = 2, 4, 2, 70, 16
+    Q, K, V = rand_bits(30, (B, Hq, N, d)), rand_bits(31, (B, Hkv, N, d)), rand_bits(32, (B, Hkv, N, d))
+    full = oracle.delta_attn(Q, K, V, 3, 11, 9, lib=lib)
+    rng = np.random.default_rng(0)
+    bhi = np.stack([rng.integers(0, B, 40), rng.integers(0, Hq, 40), rng.integers(0, N, 40)], 1)
+    r = oracle.rows(Q, K, V, 3, 11, 9, bhi, lib=lib)
+    for t, (b, h, i) in enumerate(bhi):
+        assert np.abs(r["A"][t] - full["A"][b, h, i]).max() <= TOL
+        assert np.abs(r["S"][t] - full["S"][b, h, i]).max() <= TOL
+        assert np.abs(r["D_sample"][t] - full["D"][b, h, i // 9]).max() <= TOL
+
+
+ALL_PINS = [pin_gamma1_is_sdpa, pin_full_window_is_sdpa, pin_zero_keys_closed_form,
+            pin_window1_no_sink, pin_constant_values, pin_mask_structure,
+            pin_sampled_rows_are_dense, pin_gqa_repeat, pin_lemma1, pin_rows_agree]
+# The brute-force restatement is listed separately: the mutant test shows the
+# other pins catch every planted mistake without it.
+BRUTE_PINS = [pin_brute_force]
