@@ -1,0 +1,138 @@
+/*
+ * delta_attn.h — C ABI of libdeltaattn.so: the Delta Attention prefill
+ * (Willette, Lee, Hwang, "Delta Attention: Fast and Accurate Sparse Attention
+ * Inference by Delta Correction", arXiv 2505.11254) on NVIDIA GB300 (sm_103a).
+ *
+ * What is computed (0-based rows; tau = 1/sqrt(d)):
+ *   Eq. 1   dense causal attention  D_i = sum_{j<=i} softmax_j(tau q_i.k_j) v_j
+ *   f*      StreamingLLM sparse attention over
+ *           W(i) = { j <= i : j < n_sink  or  j > i - window },
+ *           S_i = sum_{j in W(i)} softmax_W(tau q_i.k_j) v_j   (normalised over W(i) only)
+ *   Eq. 4   sampled query rows k*gamma, k = 0 .. n_s-1, n_s = ceil(N / gamma)
+ *   Alg. 1  Delta_k = D_{k gamma} - S_{k gamma}
+ *   Eq. 6   O_i = S_i + Delta_{floor(i/gamma)}
+ *           (on a sampled row this equals D_{k gamma}; the library writes D there)
+ * GQA: query head h reads KV head floor(h / (Hq/Hkv)).
+ *
+ * Layouts (all row-major, contiguous, device memory, 16-byte aligned):
+ *   Q, O, O_sparse     [B, Hq,  N, d]   bf16
+ *   K, V               [B, Hkv, N, d]   bf16
+ *   D_sampled, S_sampled [B, Hq, n_s, d] fp32 (row k holds sample row k*gamma)
+ * Supported: d in {64, 128}; Hq % Hkv == 0; N, gamma, window >= 1; n_sink >= 0;
+ * N <= 2^31 - 256; a device of compute capability 10.3 (GB300).
+ *
+ * Ownership and execution: the caller owns every buffer.  All calls are
+ * asynchronous on `stream` (a cudaStream_t; NULL is the legacy default stream)
+ * and never synchronise the device, except delta_attn_check().  Arguments are
+ * validated on the host before anything is launched; invalid arguments return
+ * an error and launch nothing.  Launch failures return DA_ERR_CUDA.  A kernel
+ * that gives up a bounded wait (it never should) records DA_ERR_TIMEOUT in a
+ * per-device status word that delta_attn_check() reports.  Results are
+ * deterministic: fixed merge order, no floating-point atomics.
+ */
+#ifndef DELTA_ATTN_H
+#define DELTA_ATTN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    DA_OK = 0,
+    DA_ERR_INVALID_ARG = -1,  /* bad sizes, NULL pointer, Hq % Hkv != 0 ... */
+    DA_ERR_UNSUPPORTED = -2,  /* head dim or device not supported            */
+    DA_ERR_MISALIGNED = -3,   /* a pointer is not 16-byte aligned            */
+    DA_ERR_WORKSPACE = -4,    /* workspace smaller than required             */
+    DA_ERR_CUDA = -5,         /* a CUDA runtime call or launch failed        */
+    DA_ERR_TIMEOUT = -6       /* a kernel gave up a bounded wait             */
+} da_status;
+
+/* Workspace bytes delta_attn_prefill() needs for this shape on the current
+ * device (fp32 dense sampled rows, Delta rows when gamma does not divide 128,
+ * split-K partials and their tickets).  Writes *bytes; returns a da_status. */
+int delta_attn_workspace_size(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma,
+                              size_t* bytes);
+
+/* The full prefill (Alg. 1 with Eq. 6): writes O.  Runs the strided dense
+ * kernel (D at the sampled rows), then the sink+window kernel whose epilogue
+ * adds Delta and writes bf16 O once.  gamma = 1 makes every row a dense row
+ * (plain causal attention).  `workspace` (device, >= the size above) may be
+ * NULL, in which case the library allocates it stream-ordered
+ * (cudaMallocAsync / cudaFreeAsync on `stream`). */
+int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
+                       int d, int n_sink, int64_t window, int gamma, void* workspace, size_t ws_bytes,
+                       void* stream);
+
+/* f*(Q,K,V) of Alg. 1 alone: StreamingLLM sink + window attention of every
+ * row, written as bf16 to O_sparse.  When S_sampled is not NULL the fp32
+ * sparse rows at the sampled rows k*gamma are also written (the operand
+ * delta_apply() subtracts). */
+int sparse_window_attn(const void* Q, const void* K, const void* V, void* O_sparse, float* S_sampled, int B,
+                       int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma, void* stream);
+
+/* Workspace bytes strided_dense_attn() needs (split-K partials, tickets). */
+int strided_dense_workspace_size(int B, int Hq, int Hkv, int64_t N, int d, int gamma, size_t* bytes);
+
+/* f(~Q,K,V) of Alg. 1 alone: dense causal attention of the sampled rows
+ * k*gamma (Eq. 4), fp32, into D_sampled [B,Hq,n_s,d].  The key range is split
+ * across CTAs where that balances the GPU; partials are merged in a fixed
+ * order.  `workspace` may be NULL (stream-ordered allocation). */
+int strided_dense_attn(const void* Q, const void* K, const void* V, float* D_sampled, int B, int Hq, int Hkv,
+                       int64_t N, int d, int gamma, void* workspace, size_t ws_bytes, void* stream);
+
+/* Eq. 6 as a separate pass: O_i = bf16(S_i + D_k - S_{k gamma}) for rows that
+ * are not sampled and O_{k gamma} = bf16(D_k), with S_i read from the bf16
+ * O_sparse and S_{k gamma} from S_sampled (fp32) or, when S_sampled is NULL,
+ * from O_sparse's sampled row.  O may alias O_sparse. */
+int delta_apply(const void* O_sparse, const float* S_sampled, const float* D_sampled, void* O, int B, int Hq,
+                int64_t N, int d, int gamma, void* stream);
+
+/* Synchronises `stream`, returns and clears the device status word
+ * (DA_OK, DA_ERR_TIMEOUT), or DA_ERR_CUDA if the stream reports an error. */
+int delta_attn_check(void* stream);
+
+/* Static description of a status code. */
+const char* delta_attn_status_string(int status);
+
+/* ---- Introspection for tests (same code paths the kernels use). ---- */
+
+/* Host: how the prefill is decomposed.  info[0..9] = CTAs of the sink+window
+ * kernel, CTAs of the strided dense kernel, CTAs of the strided sparse kernel
+ * (0 unless used), key tiles per split-K unit, split units, heads packed per
+ * sampled-row tile, samples per head in it, 1 if Delta is fused inside the
+ * row tile (gamma divides 128), kernels one prefill launches, SM count. */
+int delta_attn_plan_info(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma,
+                         int64_t* info);
+
+/* Device: out[(i - i0) * N + j] = 1 if key j is in W(i), else 0, for
+ * i in [i0, i1) — the predicate the sparse kernels apply. out: uint8 device. */
+int delta_attn_debug_mask(int64_t N, int n_sink, int64_t window, int64_t i0, int64_t i1, uint8_t* out,
+                          void* stream);
+
+/* Device: sample_row[i] = floor(i/gamma)*gamma and is_sampled[i] = (i % gamma == 0)
+ * for i in [0, N), as the epilogues compute them. */
+int delta_attn_debug_rowmap(int64_t N, int gamma, int64_t* sample_row, uint8_t* is_sampled, void* stream);
+
+/* Device: the work item `index` of kernel `mode` (0 sink+window rows,
+ * 1 strided dense, 2 strided sparse) as the kernel decodes it.  out (int64,
+ * device) holds 16 + 4*128 + 2*max_tiles entries: a header (b, first head,
+ * kv head, first row or sample, last row or sample, sink tiles, first and last
+ * band tile, tiles, chunks, chunk index, first unit, unit), then per TMEM lane
+ * (row, sample, head, valid), then per key tile (tile index, needs mask). */
+int delta_attn_debug_work(int mode, int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window,
+                          int gamma, int64_t index, int64_t* out, int max_tiles, void* stream);
+
+/* Device: exercises the bounded-wait failure path without faulting the GPU.
+ * Launches one warp that waits on an mbarrier nothing arrives on; after
+ * limit_ns (0 < limit_ns <= 1e9) the wait gives up and records DA_ERR_TIMEOUT,
+ * which the next delta_attn_check() returns (and clears). */
+int delta_attn_debug_timeout(int64_t limit_ns, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DELTA_ATTN_H */

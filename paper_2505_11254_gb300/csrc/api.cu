@@ -1,0 +1,447 @@
+// api.cu — the C ABI of libdeltaattn.so (declared in include/delta_attn.h):
+// argument validation, workspace planning, TMA descriptor encoding and the
+// launch sequence of the Delta Attention prefill (arXiv 2505.11254, Alg. 1).
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <algorithm>
+#include <cmath>
+
+#include "delta_attn.h"
+#include "launch.h"
+#include "tiles.cuh"
+#include "wait.cuh"
+
+using namespace da;
+
+// Per-device status word written by kernels that give up a bounded wait.
+__device__ int g_da_status;
+
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      p = nullptr;
+    return reinterpret_cast<EncodeTiledFn>(p);
+  }();
+  return fn;
+}
+
+// 3-D bf16 tensor map, 128-byte swizzle, boxes of 64 x box1 x box2 elements.
+// dim0 = d (contiguous), dim1 stride and dim2 stride in bytes.
+bool make_map(CUtensorMap* m, const void* base, long long d, long long dim1, long long stride1, long long dim2,
+              long long stride2, int box1, int box2) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)dim1, (cuuint64_t)dim2};
+  cuuint64_t strides[2] = {(cuuint64_t)stride1, (cuuint64_t)stride2};
+  cuuint32_t box[3] = {64, (cuuint32_t)box1, (cuuint32_t)box2};
+  cuuint32_t es[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int check_device(int* sms) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return DA_ERR_CUDA;
+  int major = 0, minor = 0;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return DA_ERR_CUDA;
+  if (major != 10 || minor != 3) return DA_ERR_UNSUPPORTED;
+  return DA_OK;
+}
+
+int check_shape(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma) {
+  if (B < 1 || Hq < 1 || Hkv < 1 || N < 1 || gamma < 1 || window < 1 || n_sink < 0) return DA_ERR_INVALID_ARG;
+  if (Hq % Hkv != 0) return DA_ERR_INVALID_ARG;
+  if (N > (int64_t(1) << 31) - 256) return DA_ERR_INVALID_ARG;
+  if ((int64_t)B * Hq > (int64_t(1) << 30)) return DA_ERR_INVALID_ARG;
+  if (d != 64 && d != 128) return DA_ERR_UNSUPPORTED;
+  return DA_OK;
+}
+
+struct Plan {
+  Params p;
+  bool fused_intile = false;
+  long long grid_sparse = 0, grid_dense = 0, grid_ssparse = 0;
+  size_t off_d = 0, off_delta = 0, off_part = 0, off_ticket = 0, total = 0;
+  size_t dense_part = 0, dense_ticket = 0, dense_total = 0;  // strided_dense_attn on its own
+};
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Sampled-row tiles pack Hp query heads of one KV group x R samples into the
+// 128 TMEM lanes, so the group's heads share each K/V tile.
+void packing(int G, int* Hp, int* R) {
+  int hp = 1;
+  if (G >= 2 && G <= 16 && (G & (G - 1)) == 0) hp = G;
+  *Hp = hp;
+  *R = BM / hp;
+}
+
+Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma, int sms) {
+  Plan pl;
+  Params& p = pl.p;
+  p = Params{};
+  p.B = B;
+  p.Hq = Hq;
+  p.Hkv = Hkv;
+  p.G = Hq / Hkv;
+  p.N = N;
+  p.n_sink = n_sink;
+  p.window = window;
+  p.gamma = gamma;
+  p.n_s = cdiv(N, gamma);
+  p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
+  packing(p.G, &p.Hp, &p.R);
+  p.groups_per_b = Hq / p.Hp;
+  p.mtiles = cdiv(p.n_s, p.R);
+  p.qtiles = cdiv(N, BM);
+
+  // Split-K: the chunk is chosen so that about two units per SM exist; the
+  // longest M-tiles split, short ones stay whole.
+  long long total_tiles = 0;
+  for (long long t = 0; t < p.mtiles; ++t) total_tiles += strided_dense_len(p, t);
+  total_tiles *= (long long)B * p.groups_per_b;
+  p.chunk = std::max<long long>(8, cdiv(total_tiles, 2LL * std::max(sms, 1)));
+  long long units = 0, multi = 0;
+  for (long long t = 0; t < p.mtiles; ++t) {
+    long long nc = cdiv(strided_dense_len(p, t), p.chunk);
+    units += nc;
+    if (nc > 1) multi += nc;
+  }
+  p.n_units = units * B * p.groups_per_b;
+  p.n_multi = multi * B * p.groups_per_b;
+
+  pl.grid_sparse = (long long)B * Hq * p.qtiles;
+  pl.grid_dense = p.n_units;
+  pl.fused_intile = gamma >= 2 && (BM % gamma) == 0;
+  pl.grid_ssparse = (gamma >= 2 && !pl.fused_intile) ? (long long)B * p.groups_per_b * p.mtiles : 0;
+
+  const size_t rows_bytes = (size_t)B * Hq * p.n_s * d * sizeof(float);
+  const size_t part_bytes = (size_t)p.n_multi * BM * (d + 2) * sizeof(float);
+  const size_t ticket_bytes = (size_t)p.n_multi * sizeof(int);
+  size_t off = 0;
+  if (gamma >= 2) {
+    pl.off_d = off;
+    off += align256(rows_bytes);
+    if (!pl.fused_intile) {
+      pl.off_delta = off;
+      off += align256(rows_bytes);
+    }
+  }
+  pl.off_part = off;
+  off += align256(part_bytes);
+  pl.off_ticket = off;
+  off += align256(ticket_bytes);
+  pl.total = off;
+  pl.dense_part = 0;
+  pl.dense_ticket = align256(part_bytes);
+  pl.dense_total = align256(part_bytes) + align256(ticket_bytes);
+  return pl;
+}
+
+int status_ptr(int** ptr) {
+  void* a = nullptr;
+  if (cudaGetSymbolAddress(&a, g_da_status) != cudaSuccess) return DA_ERR_CUDA;
+  *ptr = static_cast<int*>(a);
+  return DA_OK;
+}
+
+struct Maps {
+  CUtensorMap q, qs, k, v;
+};
+
+bool make_maps(Maps* m, const void* Q, const void* K, const void* V, const Params& p, int d, bool need_rows,
+               bool need_samples) {
+  const long long row_bytes = (long long)d * 2;
+  if (need_rows && !make_map(&m->q, Q, d, p.N, row_bytes, (long long)p.B * p.Hq, p.N * row_bytes, BM, 1))
+    return false;
+  if (need_samples && !make_map(&m->qs, Q, d, p.n_s, row_bytes * p.gamma, (long long)p.B * p.Hq,
+                                p.N * row_bytes, p.R, p.Hp))
+    return false;
+  if (!make_map(&m->k, K, d, p.N, row_bytes, (long long)p.B * p.Hkv, p.N * row_bytes, BN, 1)) return false;
+  if (!make_map(&m->v, V, d, p.N, row_bytes, (long long)p.B * p.Hkv, p.N * row_bytes, BN, 1)) return false;
+  return true;
+}
+
+template <int MODE, int EPI>
+cudaError_t launch(int d, const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v, const Params& p,
+                   long long grid, cudaStream_t s) {
+  if (d == 64) return launch_attn<64, MODE, EPI>(q, k, v, p, grid, s);
+  return launch_attn<128, MODE, EPI>(q, k, v, p, grid, s);
+}
+
+class ScopedWorkspace {
+ public:
+  ScopedWorkspace(void* user, size_t bytes, cudaStream_t s) : s_(s) {
+    if (user != nullptr || bytes == 0) {
+      ptr_ = user;
+      return;
+    }
+    if (cudaMallocAsync(&ptr_, bytes, s) != cudaSuccess) ptr_ = nullptr;
+    owned_ = ptr_ != nullptr;
+    failed_ = !owned_;
+  }
+  ~ScopedWorkspace() {
+    if (owned_) cudaFreeAsync(ptr_, s_);
+  }
+  bool failed() const { return failed_; }
+  uint8_t* get() const { return static_cast<uint8_t*>(ptr_); }
+
+ private:
+  void* ptr_ = nullptr;
+  cudaStream_t s_;
+  bool owned_ = false, failed_ = false;
+};
+
+}  // namespace
+
+extern "C" {
+
+const char* delta_attn_status_string(int status) {
+  switch (status) {
+    case DA_OK: return "ok";
+    case DA_ERR_INVALID_ARG: return "invalid argument";
+    case DA_ERR_UNSUPPORTED: return "unsupported head dimension or device (needs d in {64,128} and sm_103)";
+    case DA_ERR_MISALIGNED: return "pointer not 16-byte aligned";
+    case DA_ERR_WORKSPACE: return "workspace too small";
+    case DA_ERR_CUDA: return "CUDA error";
+    case DA_ERR_TIMEOUT: return "kernel gave up a bounded wait";
+    default: return "unknown status";
+  }
+}
+
+int delta_attn_workspace_size(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma,
+                              size_t* bytes) {
+  if (!bytes) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
+  if (rc) return rc;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  *bytes = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms).total;
+  return DA_OK;
+}
+
+int strided_dense_workspace_size(int B, int Hq, int Hkv, int64_t N, int d, int gamma, size_t* bytes) {
+  if (!bytes) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N, d, 0, 1, gamma);
+  if (rc) return rc;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  *bytes = make_plan(B, Hq, Hkv, N, d, 0, 1, gamma, sms).dense_total;
+  return DA_OK;
+}
+
+int delta_attn_plan_info(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma,
+                         int64_t* info) {
+  if (!info) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
+  if (rc) return rc;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms);
+  info[0] = gamma == 1 ? 0 : pl.grid_sparse;
+  info[1] = pl.grid_dense;
+  info[2] = pl.grid_ssparse;
+  info[3] = pl.p.chunk;
+  info[4] = pl.p.n_multi;
+  info[5] = pl.p.Hp;
+  info[6] = pl.p.R;
+  info[7] = pl.fused_intile ? 1 : 0;
+  info[8] = gamma == 1 ? 1 : (pl.fused_intile ? 2 : 3);
+  info[9] = sms;
+  return DA_OK;
+}
+
+int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
+                       int d, int n_sink, int64_t window, int gamma, void* workspace, size_t ws_bytes,
+                       void* stream) {
+  if (!Q || !K || !V || !O) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
+  if (rc) return rc;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(workspace))
+    return DA_ERR_MISALIGNED;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms);
+  if (workspace != nullptr && ws_bytes < pl.total) return DA_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Params p = pl.p;
+  if ((rc = status_ptr(&p.err))) return rc;
+  Maps m;
+  if (!make_maps(&m, Q, K, V, p, d, gamma >= 2, true)) return DA_ERR_INVALID_ARG;
+
+  ScopedWorkspace ws(workspace, pl.total, s);
+  if (ws.failed()) return DA_ERR_CUDA;
+  uint8_t* base = ws.get();
+  p.partials = reinterpret_cast<float*>(base + pl.off_part);
+  p.tickets = reinterpret_cast<int*>(base + pl.off_ticket);
+  if (p.n_multi > 0 && cudaMemsetAsync(p.tickets, 0, p.n_multi * sizeof(int), s) != cudaSuccess)
+    return DA_ERR_CUDA;
+
+  cudaError_t e;
+  if (gamma == 1) {
+    // Every row is a sampled row: the output is dense causal attention.
+    p.out_bf16 = O;
+    e = launch<MODE_STRIDED_DENSE, EPI_DENSE_BF16>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
+    return e == cudaSuccess ? DA_OK : DA_ERR_CUDA;
+  }
+  float* dbuf = reinterpret_cast<float*>(base + pl.off_d);
+  p.d_out = dbuf;
+  e = launch<MODE_STRIDED_DENSE, EPI_DENSE_F32>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
+  if (e != cudaSuccess) return DA_ERR_CUDA;
+  p.d_out = nullptr;
+  p.d_in = dbuf;
+  p.out_bf16 = O;
+  if (pl.fused_intile) {
+    e = launch<MODE_SPARSE, EPI_FUSED_INTILE>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+  } else {
+    float* delta = reinterpret_cast<float*>(base + pl.off_delta);
+    p.delta_out = delta;
+    e = launch<MODE_STRIDED_SPARSE, EPI_DELTA_BUILD>(d, m.qs, m.k, m.v, p, pl.grid_ssparse, s);
+    if (e != cudaSuccess) return DA_ERR_CUDA;
+    p.delta_out = nullptr;
+    p.delta_in = delta;
+    e = launch<MODE_SPARSE, EPI_FUSED_DELTA>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+  }
+  return e == cudaSuccess ? DA_OK : DA_ERR_CUDA;
+}
+
+int sparse_window_attn(const void* Q, const void* K, const void* V, void* O_sparse, float* S_sampled, int B,
+                       int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma, void* stream) {
+  if (!Q || !K || !V || !O_sparse) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
+  if (rc) return rc;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O_sparse) || !aligned16(S_sampled))
+    return DA_ERR_MISALIGNED;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms);
+  Params p = pl.p;
+  if ((rc = status_ptr(&p.err))) return rc;
+  Maps m;
+  if (!make_maps(&m, Q, K, V, p, d, true, false)) return DA_ERR_INVALID_ARG;
+  p.out_bf16 = O_sparse;
+  p.s_sampled = S_sampled;
+  cudaError_t e = launch<MODE_SPARSE, EPI_BF16>(d, m.q, m.k, m.v, p, pl.grid_sparse, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? DA_OK : DA_ERR_CUDA;
+}
+
+int strided_dense_attn(const void* Q, const void* K, const void* V, float* D_sampled, int B, int Hq, int Hkv,
+                       int64_t N, int d, int gamma, void* workspace, size_t ws_bytes, void* stream) {
+  if (!Q || !K || !V || !D_sampled) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N, d, 0, 1, gamma);
+  if (rc) return rc;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(D_sampled) || !aligned16(workspace))
+    return DA_ERR_MISALIGNED;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  Plan pl = make_plan(B, Hq, Hkv, N, d, 0, 1, gamma, sms);
+  if (workspace != nullptr && ws_bytes < pl.dense_total) return DA_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Params p = pl.p;
+  if ((rc = status_ptr(&p.err))) return rc;
+  Maps m;
+  if (!make_maps(&m, Q, K, V, p, d, false, true)) return DA_ERR_INVALID_ARG;
+  ScopedWorkspace ws(workspace, pl.dense_total, s);
+  if (ws.failed()) return DA_ERR_CUDA;
+  p.partials = reinterpret_cast<float*>(ws.get() + pl.dense_part);
+  p.tickets = reinterpret_cast<int*>(ws.get() + pl.dense_ticket);
+  if (p.n_multi > 0 && cudaMemsetAsync(p.tickets, 0, p.n_multi * sizeof(int), s) != cudaSuccess)
+    return DA_ERR_CUDA;
+  p.d_out = D_sampled;
+  cudaError_t e = launch<MODE_STRIDED_DENSE, EPI_DENSE_F32>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
+  return e == cudaSuccess ? DA_OK : DA_ERR_CUDA;
+}
+
+int delta_apply(const void* O_sparse, const float* S_sampled, const float* D_sampled, void* O, int B, int Hq,
+                int64_t N, int d, int gamma, void* stream) {
+  if (!O_sparse || !D_sampled || !O) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hq, N, d, 0, 1, gamma);
+  if (rc) return rc;
+  if (!aligned16(O_sparse) || !aligned16(S_sampled) || !aligned16(D_sampled) || !aligned16(O))
+    return DA_ERR_MISALIGNED;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  cudaError_t e = launch_delta_apply(O_sparse, S_sampled, D_sampled, O, B, Hq, N, d, gamma,
+                                     static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? DA_OK : DA_ERR_CUDA;
+}
+
+int delta_attn_check(void* stream) {
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return DA_ERR_CUDA;
+  int v = 0;
+  if (cudaMemcpyFromSymbolAsync(&v, g_da_status, sizeof(int), 0, cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return DA_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return DA_ERR_CUDA;
+  if (v != 0) {
+    const int zero = 0;
+    if (cudaMemcpyToSymbolAsync(g_da_status, &zero, sizeof(int), 0, cudaMemcpyHostToDevice, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+      return DA_ERR_CUDA;
+  }
+  return v;
+}
+
+int delta_attn_debug_mask(int64_t N, int n_sink, int64_t window, int64_t i0, int64_t i1, uint8_t* out,
+                          void* stream) {
+  if (!out || N < 1 || window < 1 || n_sink < 0 || i0 < 0 || i1 <= i0 || i1 > N) return DA_ERR_INVALID_ARG;
+  return launch_debug_mask(N, n_sink, window, i0, i1, out, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? DA_OK
+             : DA_ERR_CUDA;
+}
+
+int delta_attn_debug_rowmap(int64_t N, int gamma, int64_t* sample_row, uint8_t* is_sampled, void* stream) {
+  if (!sample_row || !is_sampled || N < 1 || gamma < 1) return DA_ERR_INVALID_ARG;
+  return launch_debug_rowmap(N, gamma, reinterpret_cast<long long*>(sample_row), is_sampled,
+                             static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? DA_OK
+             : DA_ERR_CUDA;
+}
+
+int delta_attn_debug_work(int mode, int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window,
+                          int gamma, int64_t index, int64_t* out, int max_tiles, void* stream) {
+  if (!out || max_tiles < 0 || mode < 0 || mode > 2) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
+  if (rc) return rc;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms);
+  const long long count = mode == 0 ? pl.grid_sparse : mode == 1 ? pl.grid_dense
+                                                                 : (long long)B * pl.p.groups_per_b * pl.p.mtiles;
+  if (index < 0 || index >= count) return DA_ERR_INVALID_ARG;
+  return launch_debug_work(mode, pl.p, index, reinterpret_cast<long long*>(out), max_tiles,
+                           static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? DA_OK
+             : DA_ERR_CUDA;
+}
+
+int delta_attn_debug_timeout(int64_t limit_ns, void* stream) {
+  if (limit_ns <= 0 || limit_ns > (int64_t)WAIT_LIMIT_NS) return DA_ERR_INVALID_ARG;
+  int* status = nullptr;
+  int rc = status_ptr(&status);
+  if (rc) return rc;
+  return launch_debug_timeout(status, (unsigned long long)limit_ns, static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? DA_OK
+             : DA_ERR_CUDA;
+}
+
+}  // extern "C"

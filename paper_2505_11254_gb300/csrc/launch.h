@@ -1,0 +1,27 @@
+// launch.h — host-side declarations of the kernel launchers (instantiated in
+// attn_*.cu so the kernels compile in parallel translation units).
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "tiles.cuh"
+
+namespace da {
+
+template <int D, int MODE, int EPI>
+cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
+                        long long grid, cudaStream_t s);
+
+unsigned attn_smem_bytes(int d);
+
+cudaError_t launch_delta_apply(const void* o_sparse, const float* s_sampled, const float* d_sampled, void* o, int B,
+                               int Hq, long long N, int d, int gamma, cudaStream_t s);
+cudaError_t launch_debug_mask(long long N, int n_sink, long long window, long long i0, long long i1,
+                              unsigned char* out, cudaStream_t s);
+cudaError_t launch_debug_rowmap(long long N, int gamma, long long* sample_row, unsigned char* sampled,
+                                cudaStream_t s);
+cudaError_t launch_debug_timeout(int* status, unsigned long long limit_ns, cudaStream_t s);
+cudaError_t launch_debug_work(int mode, const Params& p, long long index, long long* out, int max_tiles,
+                              cudaStream_t s);
+
+}  // namespace da

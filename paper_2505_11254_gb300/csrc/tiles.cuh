@@ -1,0 +1,226 @@
+// tiles.cuh — work decomposition, key-tile lists and visibility predicates of
+// the Delta Attention prefill kernels.  Used by the attention kernel and by the
+// debug kernels, so the tests check the same code the kernels run.
+//
+// Definitions (arXiv 2505.11254):
+//   * causal visibility (Eq. 1): key j is visible to query row i iff j <= i;
+//   * StreamingLLM sparse set (Sec. 2-3, f*): the first n_sink keys and the
+//     `window` most recent keys ending at i (diagonal included);
+//   * sampled rows (Eq. 4): i = k * gamma, k = 0, 1, ...; row i is corrected
+//     with the Delta of sample floor(i / gamma) (Eq. 6, Alg. 1 repeat).
+#pragma once
+#include <stdint.h>
+
+namespace da {
+
+constexpr int BM = 128;  // query rows per tile = TMEM lanes
+constexpr int BN = 128;  // keys per tile
+
+// Which rows a tile holds and which keys it visits.
+enum Mode : int {
+  MODE_SPARSE = 0,          // contiguous rows of one head, sink + window keys
+  MODE_STRIDED_DENSE = 1,   // sampled rows (GQA-packed), all causal keys, split-K
+  MODE_STRIDED_SPARSE = 2,  // sampled rows (GQA-packed), sink + window keys
+};
+
+// What the epilogue writes.
+enum Epi : int {
+  EPI_BF16 = 0,          // sparse rows -> bf16 S_i (+ fp32 S at sampled rows if requested)
+  EPI_FUSED_INTILE = 1,  // sparse rows -> bf16(S_i + D_k - S_{k gamma}), samples inside the tile
+  EPI_FUSED_DELTA = 2,   // sparse rows -> bf16(S_i + Delta_k), Delta precomputed
+  EPI_DENSE_F32 = 3,     // sampled rows -> fp32 dense rows D_k
+  EPI_DENSE_BF16 = 4,    // sampled rows (gamma = 1: every row) -> bf16 dense rows
+  EPI_DELTA_BUILD = 5,   // sampled rows -> fp32 Delta_k = D_k - S_{k gamma}
+};
+
+struct Params {
+  int B, Hq, Hkv, G;
+  long long N;
+  int n_sink;
+  long long window;
+  int gamma;
+  long long n_s;           // number of sampled rows ceil(N / gamma)
+  float scale_log2;        // log2(e) / sqrt(d)
+  // sampled-row packing: Hp heads x R samples per tile (Hp * R == BM)
+  int Hp, R;
+  int groups_per_b;        // Hq / Hp
+  long long mtiles;        // ceil(n_s / R) tiles per head group
+  long long qtiles;        // ceil(N / BM) tiles of contiguous rows per head
+  // split-K over keys for MODE_STRIDED_DENSE
+  long long chunk;         // key tiles per unit
+  long long n_units;       // units (= CTAs)
+  long long n_multi;       // leading units that belong to split M-tiles
+  // buffers
+  void* out_bf16;          // [B,Hq,N,d] bf16
+  float* s_sampled;        // [B,Hq,n_s,d] fp32, nullable
+  const float* d_in;       // [B,Hq,n_s,d] fp32 dense sampled rows (fused epilogues)
+  float* d_out;            // [B,Hq,n_s,d] fp32
+  const float* delta_in;   // [B,Hq,n_s,d] fp32
+  float* delta_out;        // [B,Hq,n_s,d] fp32
+  float* partials;         // n_multi slots of BM*(d+2) fp32
+  int* tickets;            // n_multi
+  int* err;                // device status word
+};
+
+struct Work {
+  int b, h0, g;
+  long long r0;        // MODE_SPARSE: first row; strided: first sample k0
+  long long r_last;    // last valid row / last valid sample
+  int n_sink_tiles;    // key tiles [0, n_sink_tiles) visited before the band
+  long long kt_lo;     // band tiles [kt_lo, kt_hi]
+  long long kt_hi;
+  int T;               // number of key tiles visited
+  long long unit, u0;  // split-K: this unit, first unit of its M-tile
+  int chunk_idx, n_chunks;
+};
+
+__host__ __device__ __forceinline__ long long cdiv(long long a, long long b) { return (a + b - 1) / b; }
+__host__ __device__ __forceinline__ long long lmin(long long a, long long b) { return a < b ? a : b; }
+__host__ __device__ __forceinline__ long long lmax(long long a, long long b) { return a > b ? a : b; }
+
+// --------------------------------------------------------------- predicates
+__host__ __device__ __forceinline__ bool visible_causal(long long i, long long j) { return j <= i; }
+__host__ __device__ __forceinline__ bool visible_sparse(long long i, long long j, int n_sink, long long window) {
+  return j <= i && (j < n_sink || j > i - window);
+}
+__host__ __device__ __forceinline__ long long sample_of_row(long long i, int gamma) { return (i / gamma) * gamma; }
+__host__ __device__ __forceinline__ bool is_sampled_row(long long i, int gamma) { return i % gamma == 0; }
+
+// Key tiles covering the sink keys visible to rows up to `last_row`, limited
+// to tiles before the band's first tile.
+__host__ __device__ __forceinline__ int sink_tiles_before(int n_sink, long long last_row, long long kt_lo) {
+  long long s = lmin((long long)n_sink, last_row + 1);
+  if (s <= 0) return 0;
+  return (int)lmin(kt_lo, cdiv(s, BN));
+}
+
+// Number of key tiles an M-tile of sampled rows needs under causal masking.
+__host__ __device__ __forceinline__ long long strided_dense_len(const Params& p, long long t) {
+  long long k_last = lmin(t * p.R + p.R - 1, p.n_s - 1);
+  return (k_last * p.gamma) / BN + 1;
+}
+
+// Split-K units are ordered longest-first: M-tile index t descending, then
+// (b, head group), then chunk.  Units of M-tiles with more than one chunk come
+// first because the chunk count never decreases with t.
+__host__ __device__ inline Work decode_strided_dense(const Params& p, long long unit) {
+  Work w;
+  long long per_t = (long long)p.B * p.groups_per_b;
+  long long cum = 0, t = p.mtiles - 1, nc = 1;
+  for (; t >= 0; --t) {
+    nc = cdiv(strided_dense_len(p, t), p.chunk);
+    if (unit < cum + nc * per_t) break;
+    cum += nc * per_t;
+  }
+  if (t < 0) t = 0;  // unreachable for unit < n_units
+  long long rem = unit - cum;
+  long long mt = rem / nc;
+  int c = (int)(rem % nc);
+  w.b = (int)(mt / p.groups_per_b);
+  int hg = (int)(mt % p.groups_per_b);
+  w.h0 = hg * p.Hp;
+  w.g = w.h0 / p.G;
+  w.r0 = t * p.R;
+  w.r_last = lmin(w.r0 + p.R - 1, p.n_s - 1);
+  long long L = strided_dense_len(p, t);
+  w.n_sink_tiles = 0;
+  w.kt_lo = (long long)c * p.chunk;
+  w.kt_hi = lmin(L, (long long)(c + 1) * p.chunk) - 1;
+  w.T = (int)(w.kt_hi - w.kt_lo + 1);
+  w.unit = unit;
+  w.u0 = unit - c;
+  w.chunk_idx = c;
+  w.n_chunks = (int)nc;
+  return w;
+}
+
+// Contiguous rows: CTA order is (kv-head group member fastest, q-tile, kv-head,
+// batch) so the G query heads that share K/V run side by side.
+__host__ __device__ inline Work decode_sparse(const Params& p, long long lin) {
+  Work w;
+  int hl = (int)(lin % p.G);
+  lin /= p.G;
+  long long qt = lin % p.qtiles;
+  lin /= p.qtiles;
+  w.g = (int)(lin % p.Hkv);
+  w.b = (int)(lin / p.Hkv);
+  w.h0 = w.g * p.G + hl;
+  w.r0 = qt * BM;
+  w.r_last = lmin(w.r0 + BM, p.N) - 1;
+  long long band_lo = lmax(0, w.r0 - p.window + 1);
+  w.kt_lo = band_lo / BN;
+  w.kt_hi = w.r_last / BN;
+  w.n_sink_tiles = sink_tiles_before(p.n_sink, w.r_last, w.kt_lo);
+  w.T = w.n_sink_tiles + (int)(w.kt_hi - w.kt_lo + 1);
+  w.unit = w.u0 = 0;
+  w.chunk_idx = 0;
+  w.n_chunks = 1;
+  return w;
+}
+
+// Sampled rows with the sparse key set (used when gamma does not divide BM).
+__host__ __device__ inline Work decode_strided_sparse(const Params& p, long long lin) {
+  Work w;
+  int hg = (int)(lin % p.groups_per_b);
+  lin /= p.groups_per_b;
+  long long t = lin % p.mtiles;
+  w.b = (int)(lin / p.mtiles);
+  w.h0 = hg * p.Hp;
+  w.g = w.h0 / p.G;
+  w.r0 = t * p.R;
+  w.r_last = lmin(w.r0 + p.R - 1, p.n_s - 1);
+  long long row_first = w.r0 * p.gamma, row_last = w.r_last * p.gamma;
+  w.kt_lo = lmax(0, row_first - p.window + 1) / BN;
+  w.kt_hi = row_last / BN;
+  w.n_sink_tiles = sink_tiles_before(p.n_sink, row_last, w.kt_lo);
+  w.T = w.n_sink_tiles + (int)(w.kt_hi - w.kt_lo + 1);
+  w.unit = w.u0 = 0;
+  w.chunk_idx = 0;
+  w.n_chunks = 1;
+  return w;
+}
+
+template <int MODE>
+__host__ __device__ __forceinline__ Work decode_work(const Params& p, long long lin) {
+  if (MODE == MODE_SPARSE) return decode_sparse(p, lin);
+  if (MODE == MODE_STRIDED_DENSE) return decode_strided_dense(p, lin);
+  return decode_strided_sparse(p, lin);
+}
+
+__host__ __device__ __forceinline__ long long tile_index(const Work& w, int j) {
+  return j < w.n_sink_tiles ? (long long)j : w.kt_lo + (j - w.n_sink_tiles);
+}
+
+// True when some (row, key) pair of the tile is not visible, so the kernel
+// must apply the predicate element by element.
+template <int MODE>
+__host__ __device__ __forceinline__ bool tile_needs_mask(const Params& p, const Work& w, int j) {
+  if (j < w.n_sink_tiles) return true;
+  long long kt = tile_index(w, j);
+  long long k_first = kt * BN, k_end = k_first + BN - 1;
+  if (MODE == MODE_SPARSE) {
+    return !(k_end <= w.r0 && k_first > w.r_last - p.window);
+  } else if (MODE == MODE_STRIDED_DENSE) {
+    return !(k_end <= w.r0 * p.gamma);
+  } else {
+    return !(k_end <= w.r0 * p.gamma && k_first > w.r_last * p.gamma - p.window);
+  }
+}
+
+// Query row and head of TMEM lane t.  Returns false for padding lanes.
+template <int MODE>
+__host__ __device__ __forceinline__ bool lane_row(const Params& p, const Work& w, int t, long long& row,
+                                                  long long& sample, int& head) {
+  if (MODE == MODE_SPARSE) {
+    row = w.r0 + t;
+    sample = row / p.gamma;
+    head = w.h0;
+    return row < p.N;
+  }
+  head = w.h0 + t / p.R;
+  sample = w.r0 + t % p.R;
+  row = sample * p.gamma;
+  return sample < p.n_s;
+}
+
+}  // namespace da
