@@ -1,0 +1,440 @@
+#!/usr/bin/env python
+"""Benchmark of the Delta Attention prefill on GB300 (one JSON line, rank 0).
+
+A step is one ``delta_attn_prefill`` call over one sequence of the seeded
+synthetic workload (default: Llama-3-8B-shaped attention layer, B=1, Hq=32,
+Hkv=8, d=128, N=131072, 4 sinks scaled x8, window 2048, gamma 64): the strided
+dense kernel, then the sink+window kernel with the fused Delta epilogue.
+
+  value          tokens/s of the whole job (all ranks), inputs resident in HBM
+  e2e            the same through host buffers: pinned H2D of Q,K,V, the prefill,
+                 D2H of O, every step
+  roofline       the dominant kernel's useful TFLOP/s (unmasked pairs only, 4d
+                 FLOPs per pair) against the measured bf16 peak, from CUDA events
+                 recorded by the library on the launching stream
+  cpu_baseline   the fp64 oracle on the host cores over a bounded sample
+  dense_baseline gamma = 1 through the same kernels (dense causal attention)
+
+``--impl reference`` times the oracle as the reference arm.  Multi-GPU: one
+process per GPU (torchrun), independent sequences per rank, no collective on
+the data path (weak scaling); barrier + max over ranks around the timed loop.
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from paper_2505_11254_gb300 import flops  # noqa: E402
+from paper_2505_11254_gb300.inputs import WORKLOADS, LLAMA8B_N131K, generate, to_bits  # noqa: E402
+
+METRIC = "Δ-attn prefill tokens/s and useful TFLOP/s (% bf16 tensor peak) at N=131K/1M"
+UNIT = "tokens/s"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+KERNEL_SOURCES = ["attn_kernel.cuh", "tiles.cuh", "ptx.cuh", "wait.cuh", "launch_impl.cuh"]
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=40)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=LLAMA8B_N131K.name, choices=sorted(WORKLOADS))
+    ap.add_argument("--window", type=int, default=None, help="override the workload's window")
+    ap.add_argument("--gamma", type=int, default=None, help="override the workload's gamma")
+    ap.add_argument("--cpu-seconds", type=float, default=20.0, help="oracle budget of the cpu_baseline leg")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-dense-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return dict(PEAKS_FALLBACK), "fallback"
+
+
+def kernel_src_hash():
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2505_11254_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel, workload):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current kernel source; else None."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        rec = json.load(f)
+    e = rec.get(kernel, {})
+    if e.get("src_sha") != kernel_src_hash() or e.get("workload") != workload:
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, local_index):
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        idx = str(local_index)
+        if vis:
+            parts = [p.strip() for p in vis.split(",") if p.strip()]
+            if local_index < len(parts):
+                idx = parts[local_index]
+        self.idx = idx
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits", "-i", self.idx,
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, power, reasons = [], [], [], set()
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+                power.append(float(f[3]))
+            except ValueError:
+                continue
+            for name, val in zip(self.REASONS, f[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "power_w_max": max(power) if power else None, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ dist
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------ oracle legs
+def oracle_sample(w, Qb, Kb, Vb, budget_s, max_groups=None):
+    """Time the fp64 oracle on groups of gamma rows (all query heads) at evenly
+    spaced positions of the sequence.  Returns (tokens/s, seconds, groups, cores)."""
+    import oracle
+    n_groups_total = flops.n_samples(w.N, w.gamma)
+    cores = os.cpu_count() or 1
+
+    def run(groups):
+        t0 = time.perf_counter()
+        for g in groups:
+            r0 = g * w.gamma
+            r1 = min(r0 + w.gamma, w.N)
+            oracle.delta_attn(Qb, Kb, Vb, w.n_sink, w.window, w.gamma, rows=(r0, r1), nthreads=cores)
+        return time.perf_counter() - t0
+
+    probe = [n_groups_total // 2]
+    t1 = run(probe)
+    m = max(1, int(budget_s / max(t1, 1e-6)))
+    if max_groups:
+        m = min(m, max_groups)
+    m = min(m, n_groups_total)
+    groups = sorted({int((i + 0.5) * n_groups_total / m) for i in range(m)})
+    t = run(groups)
+    rows = sum(min((g + 1) * w.gamma, w.N) - g * w.gamma for g in groups)
+    return rows * w.B / t, t, len(groups), cores
+
+
+def parity_spot_check(w, q, k, v, out, Qb, Kb, Vb):
+    """A few output rows against the oracle (sampled and unsampled rows, early
+    and late positions, the sink-dominated start)."""
+    import numpy as np
+
+    import oracle
+    N, g = w.N, w.gamma
+    rows = [0, 1, g, g + 5, N // 2, N // 2 + g - 1, N - g, N - 1]
+    bhi = [(0, h, i) for h in (0, w.Hq - 1) for i in rows]
+    ref = oracle.rows(Qb, Kb, Vb, w.n_sink, w.window, w.gamma, bhi)["A"]
+    got = np.stack([out[b, h, i].double().cpu().numpy() for (b, h, i) in bhi])
+    err = np.abs(got - ref)
+    return {"rows": len(bhi), "max_abs": float(err.max()), "mean_abs": float(err.mean()),
+            "tolerance": {"max_abs": 2e-2, "mean_abs": 2e-3}}
+
+
+# ------------------------------------------------------------------ arms
+def run_reference(args, w, world, rank):
+    """Reference arm: the fp64 CPU oracle, each step a bounded sample."""
+    if rank != 0:
+        return
+    q, k, v = generate(w, device="cpu")
+    Qb, Kb, Vb = to_bits(q), to_bits(k), to_bits(v)
+    import oracle
+    cores = os.cpu_count() or 1
+    n_groups_total = flops.n_samples(w.N, w.gamma)
+    times, rows_done = [], 0
+    for s in range(args.warmup + args.steps):
+        g = int((s * 0.618034 % 1.0) * n_groups_total)  # spread the sample over the sequence
+        r0, r1 = g * w.gamma, min(g * w.gamma + w.gamma, w.N)
+        t0 = time.perf_counter()
+        oracle.delta_attn(Qb, Kb, Vb, w.n_sink, w.window, w.gamma, rows=(r0, r1), nthreads=cores)
+        dt = time.perf_counter() - t0
+        if s >= args.warmup:
+            times.append(dt)
+            rows_done += (r1 - r0) * w.B
+    total = sum(times)
+    value = rows_done / total
+    sample = ("fp64 oracle (C, %d threads) on one group of gamma=%d rows, all %d query heads, per step, "
+              "at positions spread over the %d-token sequence" % (cores, w.gamma, w.Hq, w.N))
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * total / len(times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_of(w, args.gpus),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def config_of(w, n_gpus):
+    qkv = 2 * w.d * w.N * (w.B * w.Hq + 2 * w.B * w.Hkv)
+    l2 = ("inputs larger than L2 (Q+K+V %.2f GiB vs 129 MB L2), no flush" % (qkv / 2 ** 30) if qkv > 129e6 else
+          "inputs smaller than L2 (%.1f MB), no flush: not a headline configuration" % (qkv / 1e6))
+    return {"workload": w.name, "B": w.B, "Hq": w.Hq, "Hkv": w.Hkv, "d": w.d, "N": w.N, "n_sink": w.n_sink,
+            "window": w.window, "gamma": w.gamma, "rope_base": w.rope_base if w.rope else None,
+            "sink_scale": w.sink_scale,
+            "l2": l2,
+            "parallelism": "replicas: one independent sequence per GPU" if n_gpus > 1 else "single GPU"}
+
+
+def run_ours(args, w, world, rank, local):
+    from paper_2505_11254_gb300 import binding
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    peaks, peak_src = load_peaks()
+    wr = w.with_(seed=w.seed + rank)
+    q, k, v = generate(wr, device=dev)
+    info = binding.plan_info(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, w.gamma)
+    nk = int(info["kernels"])
+    ws = binding.alloc_workspace(binding.workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, w.gamma),
+                                 dev)
+    out = torch.empty_like(q)
+    stream = torch.cuda.current_stream()
+
+    def step(evs=None):
+        if evs is None:
+            binding.delta_attn_prefill(q, k, v, w.n_sink, w.window, w.gamma, out=out, workspace=ws)
+        else:
+            binding.delta_attn_prefill_events(q, k, v, w.n_sink, w.window, w.gamma, evs, out=out, workspace=ws)
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(args.steps)]
+    for row in evs:
+        for e in row:
+            e.record(stream)  # create the events before the timed region
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    status = binding.check()
+    if status != binding.DA_OK:
+        raise RuntimeError("device status %d after warm-up" % status)
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for s in range(args.steps):
+        step(evs[s])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clock_info = clocks.stop()
+    status = binding.check()
+    if status != binding.DA_OK:
+        raise RuntimeError("device status %d after the timed loop" % status)
+
+    elapsed_ms = max_over_ranks(t_start.elapsed_time(t_end), world)
+    ms_per_step = elapsed_ms / args.steps
+    tokens_per_step = w.B * w.N
+    value = world * tokens_per_step / (ms_per_step / 1e3)
+
+    # per-kernel durations from the library's events (launching stream)
+    names = (["strided_dense_f32", "sink_window_fused_delta"] if nk == 2 else
+             ["strided_dense_f32", "strided_sparse_delta", "sink_window_delta"] if nk == 3 else ["dense_bf16"])
+    kt = [statistics.mean(evs[s][i].elapsed_time(evs[s][i + 1]) for s in range(args.steps)) for i in range(nk)]
+    hq_flops = 4 * w.d * w.B * w.Hq
+    dense_f = hq_flops * flops.dense_pairs_per_head(w.N, w.gamma)
+    sparse_f = hq_flops * flops.sparse_pairs_per_head(w.N, w.n_sink, w.window)
+    kflops = [dense_f, sparse_f] if nk == 2 else [dense_f, 0, sparse_f] if nk == 3 else [dense_f]
+    total_f = flops.useful_flops(w.B, w.Hq, w.N, w.d, w.n_sink, w.window, w.gamma)
+    kernels = [{"name": n, "ms": t, "share": t / sum(kt), "useful_tflops": (f / (t / 1e3) / 1e12) if f else None}
+               for n, t, f in zip(names, kt, kflops)]
+    dom = max(range(nk), key=lambda i: kt[i])
+    peak = float(peaks.get("bf16_tflops", PEAKS_FALLBACK["bf16_tflops"]))
+    achieved = kflops[dom] / (kt[dom] / 1e3) / 1e12 if kflops[dom] else None
+    traffic = recorded_traffic(names[dom], w.name)
+    roofline = {"bound": "tensor", "kernel": names[dom], "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+                "peak_source": "%s bf16 dense burst (MEASURED_PEAKS.json)" % peak_src if peak_src == "measured"
+                else "fallback 1.9 PFLOP/s bf16",
+                "algorithmic": "4*d FLOPs per unmasked (query, key) pair: %.4g FLOP per launch" % kflops[dom]}
+    useful_tflops = total_f / (ms_per_step / 1e3) / 1e12
+    sustained = float(peaks.get("bf16_tflops_sustained", PEAKS_FALLBACK["bf16_tflops_sustained"]))
+
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic: seeded N(0,1) Q,K,V, RoPE base 500000 on Q,K, sink keys x%g; no dataset" % w.sink_scale,
+        "config": config_of(w, world),
+        "useful_tflops": useful_tflops, "pct_of_bf16_peak": 100 * useful_tflops / peak,
+        "pct_of_bf16_sustained": 100 * useful_tflops / sustained,
+        "roofline": roofline, "kernels": kernels, "gpu_launches": nk * args.steps,
+        "clocks": clock_info,
+    }
+
+    if not args.no_e2e:
+        # End to end through host buffers: pinned H2D of Q, K, V, the prefill,
+        # D2H of O, each step.
+        qh, kh, vh = (t.cpu().pin_memory() for t in (q, k, v))
+        oh = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
+        qd, kd, vd = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+        od = torch.empty_like(out)
+
+        def e2e_step():
+            qd.copy_(qh, non_blocking=True)
+            kd.copy_(kh, non_blocking=True)
+            vd.copy_(vh, non_blocking=True)
+            binding.delta_attn_prefill(qd, kd, vd, w.n_sink, w.window, w.gamma, out=od, workspace=ws)
+            oh.copy_(od, non_blocking=True)
+
+        for _ in range(max(1, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier(world)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1), world) / args.steps
+        if binding.check() != binding.DA_OK:
+            raise RuntimeError("device status after the e2e loop")
+        result["e2e"] = {"value": world * tokens_per_step / (e2e_ms / 1e3), "unit": UNIT,
+                         "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in (q, k, v)),
+                         "d2h_bytes_per_step": out.numel() * out.element_size(), "ms_per_step": e2e_ms}
+        del qh, kh, vh, oh, qd, kd, vd, od
+
+    if not args.no_dense_baseline and rank == 0:
+        # gamma = 1: every row dense, the same kernels (the paper's quadratic baseline)
+        dws = binding.alloc_workspace(binding.workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, 1), dev)
+        binding.delta_attn_prefill(q, k, v, w.n_sink, w.window, 1, out=out, workspace=dws)
+        torch.cuda.synchronize()
+        reps = 3
+        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        d0.record(stream)
+        for _ in range(reps):
+            binding.delta_attn_prefill(q, k, v, w.n_sink, w.window, 1, out=out, workspace=dws)
+        d1.record(stream)
+        torch.cuda.synchronize()
+        dense_ms = d0.elapsed_time(d1) / reps
+        dflops = flops.dense_flops(w.B, w.Hq, w.N, w.d)
+        result["dense_baseline"] = {"ms": dense_ms, "tflops": dflops / (dense_ms / 1e3) / 1e12,
+                                    "speedup_of_delta": dense_ms / ms_per_step,
+                                    "note": "gamma=1 through the same kernels = dense causal attention"}
+        del dws
+        step()  # restore `out` to the Delta result for the spot check
+
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        torch.cuda.synchronize()
+        Qb, Kb, Vb = to_bits(q), to_bits(k), to_bits(v)
+        result["parity"] = parity_spot_check(w, q, k, v, out, Qb, Kb, Vb)
+        tps, secs, groups, cores = oracle_sample(w, Qb, Kb, Vb, args.cpu_seconds)
+        result["cpu_baseline"] = {
+            "value": tps, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "%d groups of gamma=%d rows x all %d query heads at evenly spaced positions of the "
+                      "%d-token sequence, fp64 C oracle on %d threads, %.1f s" % (
+                          groups, w.gamma, w.Hq, w.N, cores, secs)}
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+
+
+def main():
+    args = parse_args()
+    w = WORKLOADS[args.workload]
+    if args.window is not None:
+        w = w.with_(window=args.window)
+    if args.gamma is not None:
+        w = w.with_(gamma=args.gamma)
+    world, rank, local = dist_setup(args.gpus)
+    try:
+        if args.impl == "reference":
+            run_reference(args, w, world, rank)
+        else:
+            run_ours(args, w, world, rank, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
