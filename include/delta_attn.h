@@ -66,6 +66,17 @@ int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int
                        int d, int n_sink, int64_t window, int gamma, void* workspace, size_t ws_bytes,
                        void* stream);
 
+/* delta_attn_prefill() with timing marks: records the caller's CUDA events
+ * (cudaEvent_t, created by the caller) on `stream` before the first kernel and
+ * after each kernel of the prefill, so events[i+1] - events[i] is the duration
+ * of kernel i.  n_events must equal the kernel count + 1 (plan_info()[8] + 1).
+ * The kernels are the strided dense kernel, [the strided sparse kernel when
+ * gamma does not divide 128,] and the sink+window kernel with the Delta
+ * epilogue; with gamma = 1 only the dense kernel runs. */
+int delta_attn_prefill_events(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv,
+                              int64_t N, int d, int n_sink, int64_t window, int gamma, void* workspace,
+                              size_t ws_bytes, void* stream, void* const* events, int n_events);
+
 /* f*(Q,K,V) of Alg. 1 alone: StreamingLLM sink + window attention of every
  * row, written as bf16 to O_sparse.  When S_sampled is not NULL the fp32
  * sparse rows at the sampled rows k*gamma are also written (the operand

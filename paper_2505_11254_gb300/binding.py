@@ -31,6 +31,8 @@ _sz = ctypes.c_size_t
 _SIGNATURES = {
     "delta_attn_workspace_size": ([_i, _i, _i, _i64, _i, _i, _i64, _i, ctypes.POINTER(_sz)], _i),
     "delta_attn_prefill": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _sz, _p], _i),
+    "delta_attn_prefill_events": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _sz, _p,
+                                   ctypes.POINTER(_p), _i], _i),
     "sparse_window_attn": ([_p, _p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p], _i),
     "strided_dense_workspace_size": ([_i, _i, _i, _i64, _i, _i, ctypes.POINTER(_sz)], _i),
     "strided_dense_attn": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _p, _sz, _p], _i),
@@ -125,6 +127,21 @@ def delta_attn_prefill(q, k, v, n_sink, window, gamma, out=None, workspace=None,
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check(load().delta_attn_prefill(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink, window,
                                      gamma, _dptr(workspace), ws_bytes, _stream(stream)), "delta_attn_prefill")
+    return out
+
+
+def delta_attn_prefill_events(q, k, v, n_sink, window, gamma, events, out=None, workspace=None, stream=None):
+    """The prefill with timing marks: ``events`` (torch.cuda.Event, already
+    recorded once so they exist) are recorded before the first and after each
+    kernel of the prefill on the launching stream."""
+    B, Hq, Hkv, N, d = _qkv_shape(q, k, v)
+    if out is None:
+        out = torch.empty_like(q)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    arr = (_p * len(events))(*[ctypes.c_void_p(e.cuda_event) for e in events])
+    _check(load().delta_attn_prefill_events(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink,
+                                            window, gamma, _dptr(workspace), ws_bytes, _stream(stream), arr,
+                                            len(events)), "delta_attn_prefill_events")
     return out
 
 

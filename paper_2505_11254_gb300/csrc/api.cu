@@ -269,9 +269,9 @@ int delta_attn_plan_info(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, i
   return DA_OK;
 }
 
-int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
-                       int d, int n_sink, int64_t window, int gamma, void* workspace, size_t ws_bytes,
-                       void* stream) {
+static int prefill_impl(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
+                        int d, int n_sink, int64_t window, int gamma, void* workspace, size_t ws_bytes,
+                        void* stream, void* const* events, int n_events) {
   if (!Q || !K || !V || !O) return DA_ERR_INVALID_ARG;
   int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
   if (rc) return rc;
@@ -280,6 +280,8 @@ int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int
   int sms = 0;
   if ((rc = check_device(&sms))) return rc;
   Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms);
+  const int n_kernels = gamma == 1 ? 1 : (pl.fused_intile ? 2 : 3);
+  if (n_events != 0 && (events == nullptr || n_events != n_kernels + 1)) return DA_ERR_INVALID_ARG;
   if (workspace != nullptr && ws_bytes < pl.total) return DA_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Params p = pl.p;
@@ -295,17 +297,22 @@ int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int
   if (p.n_multi > 0 && cudaMemsetAsync(p.tickets, 0, p.n_multi * sizeof(int), s) != cudaSuccess)
     return DA_ERR_CUDA;
 
+  int ev = 0;
+  auto mark = [&]() -> bool {
+    return n_events == 0 || cudaEventRecord(static_cast<cudaEvent_t>(events[ev++]), s) == cudaSuccess;
+  };
+  if (!mark()) return DA_ERR_CUDA;
   cudaError_t e;
   if (gamma == 1) {
     // Every row is a sampled row: the output is dense causal attention.
     p.out_bf16 = O;
     e = launch<MODE_STRIDED_DENSE, EPI_DENSE_BF16>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
-    return e == cudaSuccess ? DA_OK : DA_ERR_CUDA;
+    return (e == cudaSuccess && mark()) ? DA_OK : DA_ERR_CUDA;
   }
   float* dbuf = reinterpret_cast<float*>(base + pl.off_d);
   p.d_out = dbuf;
   e = launch<MODE_STRIDED_DENSE, EPI_DENSE_F32>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
-  if (e != cudaSuccess) return DA_ERR_CUDA;
+  if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
   p.d_out = nullptr;
   p.d_in = dbuf;
   p.out_bf16 = O;
@@ -315,12 +322,25 @@ int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int
     float* delta = reinterpret_cast<float*>(base + pl.off_delta);
     p.delta_out = delta;
     e = launch<MODE_STRIDED_SPARSE, EPI_DELTA_BUILD>(d, m.qs, m.k, m.v, p, pl.grid_ssparse, s);
-    if (e != cudaSuccess) return DA_ERR_CUDA;
+    if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
     p.delta_out = nullptr;
     p.delta_in = delta;
     e = launch<MODE_SPARSE, EPI_FUSED_DELTA>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
   }
-  return e == cudaSuccess ? DA_OK : DA_ERR_CUDA;
+  return (e == cudaSuccess && mark()) ? DA_OK : DA_ERR_CUDA;
+}
+
+int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
+                       int d, int n_sink, int64_t window, int gamma, void* workspace, size_t ws_bytes,
+                       void* stream) {
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, workspace, ws_bytes, stream, nullptr, 0);
+}
+
+int delta_attn_prefill_events(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv,
+                              int64_t N, int d, int n_sink, int64_t window, int gamma, void* workspace,
+                              size_t ws_bytes, void* stream, void* const* events, int n_events) {
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, workspace, ws_bytes, stream, events,
+                      n_events);
 }
 
 int sparse_window_attn(const void* Q, const void* K, const void* V, void* O_sparse, float* S_sampled, int B,
