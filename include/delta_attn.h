@@ -114,7 +114,10 @@ const char* delta_attn_status_string(int status);
  * kernel, CTAs of the strided dense kernel, CTAs of the strided sparse kernel
  * (0 unless used), key tiles per split-K unit, split units, heads packed per
  * sampled-row tile, samples per head in it, 1 if Delta is fused inside the
- * row tile (gamma divides 128), kernels one prefill launches, SM count. */
+ * row tile (gamma divides 128 and 128/gamma sampled rows fit the epilogue
+ * buffer: gamma >= 8 at d = 128, gamma >= 4 at d = 64), kernels one prefill
+ * launches, SM count.  CTA counts are work items; the kernels are persistent
+ * with min(items, SMs) CTAs. */
 int delta_attn_plan_info(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma,
                          int64_t* info);
 

@@ -130,12 +130,13 @@ Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t win
 
   pl.grid_sparse = (long long)B * Hq * p.qtiles;
   pl.grid_dense = p.n_units;
-  pl.fused_intile = gamma >= 2 && (BM % gamma) == 0;
+  pl.fused_intile = gamma >= 2 && (BM % gamma) == 0 && (size_t)(BM / gamma) * d * sizeof(float) <= kSampleBufBytes;
   pl.grid_ssparse = (gamma >= 2 && !pl.fused_intile) ? (long long)B * p.groups_per_b * p.mtiles : 0;
 
   const size_t rows_bytes = (size_t)B * Hq * p.n_s * d * sizeof(float);
   const size_t part_bytes = (size_t)p.n_multi * BM * (d + 2) * sizeof(float);
-  const size_t ticket_bytes = (size_t)p.n_multi * sizeof(int);
+  // control words zeroed before every call: 4 item counters, then the tickets
+  const size_t ticket_bytes = 4 * sizeof(unsigned long long) + (size_t)p.n_multi * sizeof(int);
   size_t off = 0;
   if (gamma >= 2) {
     pl.off_d = off;
@@ -293,8 +294,9 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   if (ws.failed()) return DA_ERR_CUDA;
   uint8_t* base = ws.get();
   p.partials = reinterpret_cast<float*>(base + pl.off_part);
-  p.tickets = reinterpret_cast<int*>(base + pl.off_ticket);
-  if (p.n_multi > 0 && cudaMemsetAsync(p.tickets, 0, p.n_multi * sizeof(int), s) != cudaSuccess)
+  p.counter = reinterpret_cast<unsigned long long*>(base + pl.off_ticket);
+  p.tickets = reinterpret_cast<int*>(base + pl.off_ticket + 4 * sizeof(unsigned long long));
+  if (cudaMemsetAsync(p.counter, 0, 4 * sizeof(unsigned long long) + p.n_multi * sizeof(int), s) != cudaSuccess)
     return DA_ERR_CUDA;
 
   int ev = 0;
@@ -382,8 +384,9 @@ int strided_dense_attn(const void* Q, const void* K, const void* V, float* D_sam
   ScopedWorkspace ws(workspace, pl.dense_total, s);
   if (ws.failed()) return DA_ERR_CUDA;
   p.partials = reinterpret_cast<float*>(ws.get() + pl.dense_part);
-  p.tickets = reinterpret_cast<int*>(ws.get() + pl.dense_ticket);
-  if (p.n_multi > 0 && cudaMemsetAsync(p.tickets, 0, p.n_multi * sizeof(int), s) != cudaSuccess)
+  p.counter = reinterpret_cast<unsigned long long*>(ws.get() + pl.dense_ticket);
+  p.tickets = reinterpret_cast<int*>(ws.get() + pl.dense_ticket + 4 * sizeof(unsigned long long));
+  if (cudaMemsetAsync(p.counter, 0, 4 * sizeof(unsigned long long) + p.n_multi * sizeof(int), s) != cudaSuccess)
     return DA_ERR_CUDA;
   p.d_out = D_sampled;
   cudaError_t e = launch<MODE_STRIDED_DENSE, EPI_DENSE_F32>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);

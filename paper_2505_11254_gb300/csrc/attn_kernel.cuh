@@ -2,20 +2,30 @@
 // of the Delta Attention prefill (arXiv 2505.11254, Alg. 1):
 //   MODE_SPARSE          f*(Q,K,V): StreamingLLM sink + window attention, every row
 //   MODE_STRIDED_DENSE   f(~Q,K,V): dense causal attention of the rows k*gamma (Eq. 4)
-//   MODE_STRIDED_SPARSE  f* at the rows k*gamma (only when gamma does not divide BM)
+//   MODE_STRIDED_SPARSE  f* at the rows k*gamma (when the Delta is not fused in-tile)
 // and the Delta epilogues (Eq. 6) that turn them into the corrected output.
 //
-// One CTA owns a 128-row query tile (TMEM lanes) and walks its key tiles.
-// Warp roles (192 threads):
-//   warps 0-3  softmax: one query row per thread; TMEM S -> P (bf16, in TMEM);
-//              lazy O rescaling; the epilogue.
-//   warp 4     TMA producer: Q once, then K and V tiles through a STAGES ring.
-//   warp 5     MMA issuer: S = Q K^T (smem x smem -> TMEM) and O += P V
-//              (TMEM x smem -> TMEM), tcgen05.commit -> mbarriers.
-// TMEM: S/P double buffer at columns [0, 2*BN), O at [2*BN, 2*BN + D).
-// Every wait is bounded: a wait that exceeds WAIT_LIMIT_NS sets the CTA's
-// abort flag and the device status word, every role leaves its loop, the CTA
-// drains its in-flight copies and MMAs, frees TMEM and returns.
+// Persistent: each CTA walks work items blockIdx.x, blockIdx.x + gridDim.x, ...
+// An item is a 128-row query tile (TMEM lanes) and its list of 128-key tiles.
+// Warp roles (384 threads = 3 warpgroups):
+//   warps 0-3  softmax: one query row per thread; S (TMEM) -> P (bf16, TMEM,
+//              aliasing S); lazy O rescaling; per item the row sum l and max m.
+//   warps 4-7  epilogue: copies the next item's Q (smem -> TMEM) ahead of time,
+//              then reads O out of TMEM, releases it, normalises, applies the
+//              Delta correction and writes the output.
+//   warp 8     TMA producer: Q of the next item, K/V tiles through a ring.
+//   warp 9     MMA issuer: S = Q K^T (Q from TMEM, K from smem) and
+//              O += P V (P from TMEM, V from smem); tcgen05.commit -> mbarriers.
+//   warps 10-11 idle (they complete the third warpgroup).
+// Registers: launched at 168 per thread (384 x 168 = 64512); the third
+// warpgroup gives back to 72 and the softmax and epilogue warpgroups grow to
+// 216, so 2 x 128 x 216 + 128 x 72 = 64512 exactly.
+// TMEM (512 columns): Q double buffer [0,64) [64,128) (bf16 pairs), S/P double
+// buffer [128,256) [256,384), O [384, 384 + D).
+// Every wait is bounded: past its limit a wait sets the CTA's abort flag and
+// the device status word, the roles stop working (keeping every named barrier
+// and warp-collective instruction uniform), drain their in-flight copies and
+// MMAs, free TMEM and return.
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -24,40 +34,82 @@
 
 #include "ptx.cuh"
 #include "tiles.cuh"
+#include "launch.h"
 #include "wait.cuh"
 
 namespace da {
 
-constexpr int kThreads = 192;
+constexpr int kThreads = 384;
+constexpr int kRegsCompute = 216;  // softmax and epilogue warpgroups
+constexpr int kRegsControl = 72;   // producer / MMA warpgroup
+static_assert(2 * 128 * kRegsCompute + 128 * kRegsControl <= kThreads * 168, "register split above the launch total");
 constexpr float RESCALE_THRESHOLD = 8.0f;  // log2 units; O is rescaled only past this
+constexpr uint32_t kFull = 0xffffffffu;
 
 template <int D>
 struct Cfg {
-  static constexpr int STAGES = (D == 128) ? 3 : 4;
-  static constexpr int CHUNKS = D / 64;                  // 64-element (128-byte) swizzle columns
+  static constexpr int NS = (D == 128) ? 5 : 8;  // K/V ring slots (one K or V tile each)
+  static constexpr int CHUNKS = D / 64;          // 64-element (128-byte) swizzle columns
   static constexpr uint32_t Q_BYTES = BM * D * 2;
   static constexpr uint32_t KV_BYTES = BN * D * 2;
-  static constexpr uint32_t SMEM = Q_BYTES + 2 * STAGES * KV_BYTES + 1024;  // + alignment slack
+  static constexpr uint32_t SBUF_BYTES = kSampleBufBytes;  // sampled sparse rows of the fused epilogue
+  static constexpr uint32_t SMEM = Q_BYTES + NS * KV_BYTES + SBUF_BYTES + 1024;
   static constexpr uint32_t TMEM_COLS = 512;
-  static constexpr uint32_t COL_O = 2 * BN;
+  static constexpr uint32_t COL_Q = 0;           // + 64 * buffer
+  static constexpr uint32_t COL_S = 128;         // + BN * buffer
+  static constexpr uint32_t COL_O = 384;
   static constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, 0, 0);
   static constexpr uint32_t IDESC_PV = idesc_bf16(BM, D, 0, 1);
 };
 
 struct Bars {
-  uint64_t q_full;
-  uint64_t k_full[4], v_full[4], k_empty[4], v_empty[4];
+  uint64_t full[8], empty[8];
+  uint64_t q_full, q_free;
+  uint64_t qt_ready[2];
   uint64_t s_full[2], p_full[2];
-  uint64_t o_done;
+  uint64_t o_step, o_full, o_free;
+  uint64_t l_ready[2], l_free[2];
   uint64_t drain;
 };
+
+template <int N>
+__device__ __forceinline__ void regs_increase() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <int N>
+__device__ __forceinline__ void regs_decrease() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
 
 __device__ __forceinline__ void named_bar_sync(int id, int n) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
 
-template <int D>
-__device__ __forceinline__ void store_row_bf16(__nv_bfloat16* dst, const float* v) {
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
+__device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float* v) {
 #pragma unroll
   for (int c = 0; c < 32; c += 8) {
     uint4 u;
@@ -91,42 +143,106 @@ __device__ __forceinline__ void load_f32x32_cg(const float* src, float* v) {
   }
 }
 
+// TMEM lane quarter of a warp: warps w and w+4 see lanes 32*(w%4) .. +31.
+__device__ __forceinline__ uint32_t lane_base(int warp) { return static_cast<uint32_t>((warp & 3) * 32) << 16; }
+
+template <int NCOL>
+__device__ __forceinline__ void tmem_ld_row(uint32_t addr, float (&v)[NCOL]) {
+#pragma unroll
+  for (int q = 0; q < NCOL / 32; ++q) {
+    uint32_t r[32];
+    tmem_ld32(addr + q * 32, r);
+#pragma unroll
+    for (int c = 0; c < 32; ++c) v[q * 32 + c] = __uint_as_float(r[c]);
+  }
+  tmem_ld_wait();
+}
+
+// Work items of a CTA.  Static: blockIdx.x, blockIdx.x + gridDim.x, ...
+// Dynamic (the split-K dense units, whose lengths differ): the producer claims
+// items from a global counter, longest first, and publishes them to the other
+// roles through a small shared-memory queue; the others read them in order.
+constexpr int kQueue = 8;
+constexpr int kQueueReaders = 9;  // MMA thread + 4 softmax warps + 4 epilogue warps
+struct ItemQueue {
+  long long item[kQueue];
+  uint64_t full[kQueue], empty[kQueue];
+};
+
+// WARP_WIDE: all 32 lanes of the warp call next() together (softmax and
+// epilogue warps); otherwise a single lane does (the MMA thread) and no
+// warp-collective instruction may be used.
+template <bool DYN, bool WARP_WIDE>
+struct ItemReader {
+  long long next_static;
+  int n = 0;
+  __device__ long long next(const Params& p, ItemQueue& q, volatile int* abort_flag) {
+    if (!DYN) {
+      const long long v = next_static;
+      next_static += gridDim.x;
+      return v < p.n_items ? v : -1;
+    }
+    const int slot = n % kQueue;
+    long long v = -1;
+    bool got = wait_bounded(&q.full[slot], (n / kQueue) & 1, abort_flag, p.err);
+    if (WARP_WIDE) got = __all_sync(kFull, got);
+    if (got) v = q.item[slot];
+    if (WARP_WIDE) {
+      __syncwarp();
+      if ((threadIdx.x & 31) == 0) mbar_arrive(&q.empty[slot]);
+    } else {
+      mbar_arrive(&q.empty[slot]);
+    }
+    ++n;
+    return v;
+  }
+};
+
 template <int D, int MODE, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const Params p) {
   using C = Cfg<D>;
-  constexpr int ST = C::STAGES;
+  constexpr int NS = C::NS;
   extern __shared__ uint8_t dsm_raw[];
   uint8_t* dsm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = dsm;
-  uint8_t* sK = sQ + C::Q_BYTES;
-  uint8_t* sV = sK + ST * C::KV_BYTES;
+  uint8_t* ring = sQ + C::Q_BYTES;
+  float* sbuf = reinterpret_cast<float*>(ring + NS * C::KV_BYTES);
 
   __shared__ Bars bars;
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_sh;
   __shared__ int ticket_sh;
+  __shared__ float lfin[2][BM], mfin[2][BM];
+  __shared__ ItemQueue iq;
+  constexpr bool DYN = (MODE == MODE_STRIDED_DENSE);
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
-  const Work w = decode_work<MODE>(p, blockIdx.x);
-  const int T = w.T;
 
   if (tid == 0) {
-    mbar_init(&bars.q_full, 1);
-    for (int s = 0; s < ST; ++s) {
-      mbar_init(&bars.k_full[s], 1);
-      mbar_init(&bars.v_full[s], 1);
-      mbar_init(&bars.k_empty[s], 1);
-      mbar_init(&bars.v_empty[s], 1);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&bars.full[s], 1);
+      mbar_init(&bars.empty[s], 1);
     }
+    mbar_init(&bars.q_full, 1);
+    mbar_init(&bars.q_free, 128);
     for (int b = 0; b < 2; ++b) {
+      mbar_init(&bars.qt_ready[b], 128);
       mbar_init(&bars.s_full[b], 1);
       mbar_init(&bars.p_full[b], 128);
+      mbar_init(&bars.l_ready[b], 128);
+      mbar_init(&bars.l_free[b], 128);
     }
-    mbar_init(&bars.o_done, 1);
+    mbar_init(&bars.o_step, 1);
+    mbar_init(&bars.o_full, 1);
+    mbar_init(&bars.o_free, 128);
     mbar_init(&bars.drain, 1);
+    for (int k = 0; k < kQueue; ++k) {
+      mbar_init(&iq.full[k], 1);
+      mbar_init(&iq.empty[k], kQueueReaders);
+    }
     abort_sh = 0;
     fence_mbar_init();
   }
@@ -139,316 +255,451 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = tmem_base_sh;
 
-  if (warp == 4) {
-    // ------------------------------------------------------------ producer
+  if (warp == 8) {
+    // ================================================================ producer
+    regs_decrease<kRegsControl>();
     if ((tid & 31) == 0) {
       prefetch_tmap(&tmQ);
       prefetch_tmap(&tmK);
       prefetch_tmap(&tmV);
-      const int qz = w.b * p.Hq + w.h0;
-      const int kz = w.b * p.Hkv + w.g;
-      mbar_arrive_expect_tx(&bars.q_full, C::Q_BYTES);
-      for (int c = 0; c < C::CHUNKS; ++c)
-        tma_load_3d(sQ + c * (BM * 128), &tmQ, &bars.q_full, c * 64, (int)w.r0, qz);
-      int nk = 0, nv = 0;  // K and V tiles issued
-      for (int j = 0; j < T; ++j) {
-        const int s = j % ST;
-        const uint32_t n = j / ST;
-        const int krow = (int)(tile_index(w, j) * BN);
-        if (j >= ST && !wait_bounded(&bars.k_empty[s], (n - 1) & 1, &abort_sh, p.err)) break;
-        mbar_arrive_expect_tx(&bars.k_full[s], C::KV_BYTES);
-        for (int c = 0; c < C::CHUNKS; ++c)
-          tma_load_3d(sK + s * C::KV_BYTES + c * (BN * 128), &tmK, &bars.k_full[s], c * 64, krow, kz);
-        ++nk;
-        if (j >= ST && !wait_bounded(&bars.v_empty[s], (n - 1) & 1, &abort_sh, p.err)) break;
-        mbar_arrive_expect_tx(&bars.v_full[s], C::KV_BYTES);
-        for (int c = 0; c < C::CHUNKS; ++c)
-          tma_load_3d(sV + s * C::KV_BYTES + c * (BN * 128), &tmV, &bars.v_full[s], c * 64, krow, kz);
-        ++nv;
+      int c = 0, nq = 0;
+      bool ok = true;
+      auto load_q = [&](long long item) {
+        const Work wq = decode_work<MODE>(p, item);
+        if (nq >= 1 && !wait_bounded(&bars.q_free, (nq - 1) & 1, &abort_sh, p.err)) return false;
+        mbar_arrive_expect_tx(&bars.q_full, C::Q_BYTES);
+        for (int ch = 0; ch < C::CHUNKS; ++ch)
+          tma_load_3d(sQ + ch * (BM * 128), &tmQ, &bars.q_full, ch * 64, (int)wq.r0, wq.b * p.Hq + wq.h0);
+        ++nq;
+        return true;
+      };
+      auto load_kv = [&](const CUtensorMap* m, int row, int z) {
+        const int s = c % NS;
+        if (c >= NS && !wait_bounded(&bars.empty[s], ((c / NS) - 1) & 1, &abort_sh, p.err)) return false;
+        mbar_arrive_expect_tx(&bars.full[s], C::KV_BYTES);
+        for (int ch = 0; ch < C::CHUNKS; ++ch)
+          tma_load_3d(ring + s * C::KV_BYTES + ch * (BN * 128), m, &bars.full[s], ch * 64, row, z);
+        ++c;
+        return true;
+      };
+      // Claims the next item (or -1) and, when dynamic, publishes it.
+      long long next_static = blockIdx.x;
+      int np = 0;
+      bool done = false;
+      auto claim = [&]() -> long long {
+        long long v = -1;
+        if (!done) {
+          if (DYN) {
+            v = (long long)atomicAdd(p.counter, 1ull);
+          } else {
+            v = next_static;
+            next_static += gridDim.x;
+          }
+          if (v >= p.n_items) v = -1;
+        }
+        if (DYN && !done) {
+          const int slot = np % kQueue;
+          if (np >= kQueue && !wait_bounded(&iq.empty[slot], ((np / kQueue) - 1) & 1, &abort_sh, p.err)) v = -1;
+          iq.item[slot] = v;
+          mbar_arrive(&iq.full[slot]);
+          ++np;
+        }
+        done = done || v < 0;
+        return v;
+      };
+      long long item = claim();
+      if (item >= 0) ok = load_q(item);
+      while (ok && item >= 0) {
+        const Work w = decode_work<MODE>(p, item);
+        const int kz = w.b * p.Hkv + w.g;
+        long long nxt = -1;
+        for (int j = 0; ok && j < w.T; ++j) {
+          const int krow = (int)(tile_index(w, j) * BN);
+          ok = load_kv(&tmK, krow, kz) && load_kv(&tmV, krow, kz);
+          if (ok && j == 0) {
+            nxt = claim();
+            if (nxt >= 0) ok = load_q(nxt);
+          }
+        }
+        item = nxt;
       }
-      // Drain: every copy lands before the CTA exits.  Copies older than the
-      // last ST per ring were consumed (their stage was reused), so only the
-      // last ST can be in flight; in the normal path they have landed already.
-      for (int jj = (nk > ST ? nk - ST : 0); jj < nk; ++jj) wait_drain(&bars.k_full[jj % ST], (jj / ST) & 1, p.err);
-      for (int jj = (nv > ST ? nv - ST : 0); jj < nv; ++jj) wait_drain(&bars.v_full[jj % ST], (jj / ST) & 1, p.err);
-      wait_drain(&bars.q_full, 0, p.err);
+      if (DYN && !done) claim();  // the readers always see the end of the sequence
+      // Drain: only the last NS ring loads and the last Q load can be in flight.
+      for (int u = (c > NS ? c - NS : 0); u < c; ++u) wait_drain(&bars.full[u % NS], (u / NS) & 1, p.err);
+      if (nq > 0) wait_drain(&bars.q_full, (nq - 1) & 1, p.err);
     }
-  } else if (warp == 5) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 9) {
+    // ================================================================ MMA issuer
+    regs_decrease<kRegsControl>();
     if ((tid & 31) == 0) {
-      const uint32_t q_base = smem_u32(sQ);
-      const uint32_t k_base = smem_u32(sK);
-      const uint32_t v_base = smem_u32(sV);
-      bool ok = wait_bounded(&bars.q_full, 0, &abort_sh, p.err);
-      tc_fence_after();
-      for (int j = 0; ok && j <= T; ++j) {
-        if (j < T) {
-          const int s = j % ST;
-          const uint32_t sb = (j & 1) * BN;
-          if (!wait_bounded(&bars.k_full[s], (j / ST) & 1, &abort_sh, p.err)) break;
-          tc_fence_after();
+      const uint32_t ring_base = smem_u32(ring);
+      int c = 0;
+      long long g = 0;
+      bool ok = true;
+      struct Pend {
+        long long g;
+        int vslot, item_i;
+        uint32_t vph;
+        bool first, last;
+      } pend{0, 0, 0, 0, false, false};
+      bool has_pend = false;
+      auto issue_pv = [&](const Pend& pv) {
+        if (!wait_bounded(&bars.p_full[pv.g & 1], (pv.g >> 1) & 1, &abort_sh, p.err)) return false;
+        if (!wait_bounded(&bars.full[pv.vslot], pv.vph, &abort_sh, p.err)) return false;
+        if (pv.first && pv.item_i >= 1 && !wait_bounded(&bars.o_free, (pv.item_i - 1) & 1, &abort_sh, p.err))
+          return false;
+        tc_fence_after();
+        const uint32_t sb = tmem + C::COL_S + (uint32_t)(pv.g & 1) * BN;
+        const uint32_t vb = ring_base + pv.vslot * C::KV_BYTES;
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * (BM * 128) + (kk & 3) * 32;
-            const uint32_t koff = (kk >> 2) * (BN * 128) + (kk & 3) * 32;
-            mma_ss(tmem + sb, sdesc_sw128(q_base + off, 16, 1024),
-                   sdesc_sw128(k_base + s * C::KV_BYTES + koff, 16, 1024), C::IDESC_QK, kk > 0);
-          }
-          mma_commit(&bars.s_full[j & 1]);
-          mma_commit(&bars.k_empty[s]);
-        }
-        if (j >= 1) {
-          const int jp = j - 1;
-          const int s = jp % ST;
-          const uint32_t sb = (jp & 1) * BN;
-          if (!wait_bounded(&bars.p_full[jp & 1], (jp >> 1) & 1, &abort_sh, p.err)) break;
-          if (!wait_bounded(&bars.v_full[s], (jp / ST) & 1, &abort_sh, p.err)) break;
+        for (int kk = 0; kk < BN / 16; ++kk)
+          mma_ts(tmem + C::COL_O, sb + kk * 8, sdesc_sw128(vb + kk * 2048, BN * 128, 1024), C::IDESC_PV,
+                 (pv.first && kk == 0) ? 0u : 1u);
+        mma_commit(&bars.o_step);
+        mma_commit(&bars.empty[pv.vslot]);
+        if (pv.last) mma_commit(&bars.o_full);
+        return true;
+      };
+      ItemReader<DYN, false> items{(long long)blockIdx.x};
+      int i = 0;
+      for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
+        const Work w = decode_work<MODE>(p, item);
+        if (!wait_bounded(&bars.qt_ready[i & 1], (i >> 1) & 1, &abort_sh, p.err)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t qt = tmem + C::COL_Q + (uint32_t)(i & 1) * 64;
+        for (int j = 0; j < w.T; ++j) {
+          const int ks = c % NS;
+          const uint32_t kph = (c / NS) & 1;
+          ++c;
+          const int vs = c % NS;
+          const uint32_t vph = (c / NS) & 1;
+          ++c;
+          if (!wait_bounded(&bars.full[ks], kph, &abort_sh, p.err)) { ok = false; break; }
           tc_fence_after();
+          const uint32_t sb = tmem + C::COL_S + (uint32_t)(g & 1) * BN;
+          const uint32_t kb = ring_base + ks * C::KV_BYTES;
 #pragma unroll
-          for (int kk = 0; kk < BN / 16; ++kk) {
-            mma_ts(tmem + C::COL_O, tmem + sb + kk * 8,
-                   sdesc_sw128(v_base + s * C::KV_BYTES + kk * 2048, BN * 128, 1024), C::IDESC_PV,
-                   (jp > 0 || kk > 0) ? 1u : 0u);
-          }
-          mma_commit(&bars.o_done);
-          mma_commit(&bars.v_empty[s]);
+          for (int kk = 0; kk < D / 16; ++kk)
+            mma_ts(sb, qt + kk * 8, sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024),
+                   C::IDESC_QK, kk > 0 ? 1u : 0u);
+          mma_commit(&bars.s_full[g & 1]);
+          mma_commit(&bars.empty[ks]);
+          if (has_pend && !issue_pv(pend)) { ok = false; break; }
+          pend = Pend{g, vs, i, vph, j == 0, j == w.T - 1};
+          has_pend = true;
+          ++g;
         }
       }
+      if (ok && has_pend) issue_pv(pend);
       // Drain: all MMAs issued by this thread complete before TMEM is freed.
       mma_commit(&bars.drain);
       wait_drain(&bars.drain, 0, p.err);
     }
-  } else {
-    // ------------------------------------------------------------ softmax
-    const int t = tid;  // TMEM lane = query row of the tile
-    const uint32_t lane_addr = static_cast<uint32_t>(warp * 32) << 16;
-    long long row, sample;
-    int head;
-    const bool row_ok = lane_row<MODE>(p, w, t, row, sample, head);
-    float m_run = -INFINITY, l_run = 0.f;
+  } else if (warp >= 10) {
+    // idle warps of the control warpgroup
+    regs_decrease<kRegsControl>();
+  } else if (warp < 4) {
+    // ================================================================ softmax
+    regs_increase<kRegsCompute>();
+    const int t = tid;
+    const uint32_t la = lane_base(warp);
+    const float scale = p.scale_log2;
+    const uint64_t scale2 = f2_pack(scale, scale);
+    long long g = 0;
     bool ok = true;
-    for (int j = 0; j < T && ok; ++j) {
-      const uint32_t sb = (j & 1) * BN;
-      if (!__all_sync(0xffffffffu, wait_bounded(&bars.s_full[j & 1], (j >> 1) & 1, &abort_sh, p.err))) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      float x[BN];
-#pragma unroll
-      for (int q = 0; q < BN / 32; ++q) {
-        uint32_t r[32];
-        tmem_ld32(tmem + lane_addr + sb + q * 32, r);
-        tmem_ld_wait();
-#pragma unroll
-        for (int c = 0; c < 32; ++c) x[q * 32 + c] = __uint_as_float(r[c]) * p.scale_log2;
-      }
-      if (tile_needs_mask<MODE>(p, w, j)) {
-        const long long k0 = tile_index(w, j) * BN;
-#pragma unroll
-        for (int c = 0; c < BN; ++c) {
-          const long long key = k0 + c;
-          const bool vis = (MODE == MODE_STRIDED_DENSE) ? visible_causal(row, key)
-                                                        : visible_sparse(row, key, p.n_sink, p.window);
-          if (!vis) x[c] = -INFINITY;
+    int i = 0;
+    ItemReader<DYN, true> items{(long long)blockIdx.x};
+    for (long long item = items.next(p, iq, &abort_sh); item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
+      const Work w = decode_work<MODE>(p, item);
+      long long row, sample;
+      int head;
+      lane_row<MODE>(p, w, t, row, sample, head);
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; ok && j < w.T; ++j, ++g) {
+        if (!__all_sync(kFull, wait_bounded(&bars.s_full[g & 1], (g >> 1) & 1, &abort_sh, p.err))) {
+          ok = false;
+          break;
         }
-      }
-      float mt = x[0];
-#pragma unroll
-      for (int c = 1; c < BN; ++c) mt = fmaxf(mt, x[c]);
-      float m_use = m_run;
-      bool rescale = false;
-      if (m_run == -INFINITY) {
-        m_use = mt;
-        rescale = (j > 0) && (mt != -INFINITY);  // O holds zeros; scaling by 0 keeps it so
-      } else if (mt > m_run + RESCALE_THRESHOLD) {
-        m_use = mt;
-        rescale = true;
-      }
-      const float m_base = (m_use == -INFINITY) ? 0.f : m_use;
-      float l_tile = 0.f;
-      uint32_t pk[BN / 2];
-#pragma unroll
-      for (int c = 0; c < BN; c += 2) {
-        const float p0 = ex2(x[c] - m_base), p1 = ex2(x[c + 1] - m_base);
-        l_tile += p0 + p1;
-        pk[c / 2] = pack_bf16x2(p0, p1);
-      }
-      // PV(j-1) must be complete before O is rescaled and before P(j)
-      // overwrites the buffer that P(j-2) used (in-order MMA completion).
-      if (j >= 1 && !__all_sync(0xffffffffu, wait_bounded(&bars.o_done, (j - 1) & 1, &abort_sh, p.err))) {
-        ok = false;
-        break;
-      }
-      // tcgen05.ld/st are warp-collective: the warp rescales together, rows
-      // that need no rescale use the factor 1.
-      if (__any_sync(0xffffffffu, rescale)) {
-        const float f = !rescale ? 1.f : (m_run == -INFINITY) ? 0.f : ex2(m_run - m_use);
-        l_run *= f;
         tc_fence_after();
+        const uint32_t sb = C::COL_S + (uint32_t)(g & 1) * BN;
+        float s[BN];
+        tmem_ld_row<BN>(tmem + la + sb, s);
+        if (tile_needs_mask<MODE>(p, w, j)) {
+          const long long k0 = tile_index(w, j) * BN;
+          const int hi = (int)lmax(-1, lmin(BN - 1, row - k0));  // causal: key offset <= hi
+          int lo = 0, se = BN;                                    // band start, sink end
+          if (MODE != MODE_STRIDED_DENSE) {
+            lo = (int)lmax(0, lmin(BN, row - p.window + 1 - k0));
+            se = (int)lmax(0, lmin(BN, (long long)p.n_sink - k0));
+          }
 #pragma unroll
-        for (int q = 0; q < D / 32; ++q) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_addr + C::COL_O + q * 32, r);
-          tmem_ld_wait();
-#pragma unroll
-          for (int c = 0; c < 32; ++c) r[c] = __float_as_uint(__uint_as_float(r[c]) * f);
-          tmem_st32(tmem + lane_addr + C::COL_O + q * 32, r);
+          for (int c = 0; c < BN; ++c) {
+            const bool vis = (c <= hi) && (c >= lo || c < se);
+            s[c] = vis ? s[c] : -INFINITY;
+          }
         }
-      }
-      l_run += l_tile;
-      m_run = m_use;
+        float mx[4];
 #pragma unroll
-      for (int q = 0; q < BN / 32; ++q) {
-        uint32_t r[16];
+        for (int q = 0; q < 4; ++q) mx[q] = s[q];
 #pragma unroll
-        for (int c = 0; c < 16; ++c) r[c] = pk[q * 16 + c];
-        tmem_st16(tmem + lane_addr + sb + q * 16, r);
+        for (int c = 4; c + 8 <= BN; c += 8) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) mx[q] = max3(mx[q], s[c + q], s[c + 4 + q]);
+        }
+        mx[0] = max3(mx[0], s[BN - 4], s[BN - 3]);
+        mx[1] = max3(mx[1], s[BN - 2], s[BN - 1]);
+        const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * scale;  // log2 units
+        float m_use = m_run;
+        bool rescale = false;
+        if (m_run == -INFINITY) {
+          m_use = mt;
+          rescale = (j > 0) && (mt != -INFINITY);  // O holds zeros; scaling by 0 keeps it so
+        } else if (mt > m_run + RESCALE_THRESHOLD) {
+          m_use = mt;
+          rescale = true;
+        }
+        const float nb = (m_use == -INFINITY) ? 0.f : -m_use;
+        const uint64_t nb2 = f2_pack(nb, nb);
+        uint64_t acc[4] = {0, 0, 0, 0};
+        uint32_t pk[BN / 2];
+#pragma unroll
+        for (int c = 0; c < BN; c += 2) {
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(s[c], s[c + 1]), scale2, nb2), x0, x1);
+          const float p0 = ex2(x0), p1 = ex2(x1);
+          acc[(c >> 1) & 3] = f2_add(acc[(c >> 1) & 3], f2_pack(p0, p1));
+          pk[c / 2] = pack_bf16x2(p0, p1);
+        }
+        float a0, a1, a2, a3, a4, a5, a6, a7;
+        f2_unpack(acc[0], a0, a1);
+        f2_unpack(acc[1], a2, a3);
+        f2_unpack(acc[2], a4, a5);
+        f2_unpack(acc[3], a6, a7);
+        const float l_tile = ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
+        // Rescale O (rare): PV(g-1) must have landed.  s_full(g) implies PV(g-2)
+        // completed, so the parity of PV(g-1) is unambiguous.
+        if (__any_sync(kFull, rescale)) {
+          if (!__all_sync(kFull, wait_bounded(&bars.o_step, (uint32_t)((g - 1) & 1), &abort_sh, p.err))) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const float f = !rescale ? 1.f : (m_run == -INFINITY) ? 0.f : ex2(m_run - m_use);
+          l_run *= f;
+#pragma unroll
+          for (int q = 0; q < D / 32; ++q) {
+            uint32_t r[32];
+            tmem_ld32(tmem + la + C::COL_O + q * 32, r);
+            tmem_ld_wait();
+#pragma unroll
+            for (int c = 0; c < 32; ++c) r[c] = __float_as_uint(__uint_as_float(r[c]) * f);
+            tmem_st32(tmem + la + C::COL_O + q * 32, r);
+          }
+        }
+        l_run += l_tile;
+        m_run = m_use;
+#pragma unroll
+        for (int q = 0; q < BN / 32; ++q) {
+          uint32_t r[16];
+#pragma unroll
+          for (int c = 0; c < 16; ++c) r[c] = pk[q * 16 + c];
+          tmem_st16(tmem + la + sb + q * 16, r);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive(&bars.p_full[g & 1]);
       }
-      tmem_st_wait();
-      tc_fence_before();
-      mbar_arrive(&bars.p_full[j & 1]);
+      if (!ok) continue;  // keep reading the item sequence to its end
+      // Publish this item's row sum and max to the epilogue.
+      if (i >= 2 && !__all_sync(kFull, wait_bounded(&bars.l_free[i & 1], ((i >> 1) - 1) & 1, &abort_sh, p.err))) {
+        ok = false;
+        continue;
+      }
+      lfin[i & 1][t] = l_run;
+      mfin[i & 1][t] = m_run;
+      mbar_arrive(&bars.l_ready[i & 1]);
     }
-    if (ok && T > 0) ok = __all_sync(0xffffffffu, wait_bounded(&bars.o_done, (T - 1) & 1, &abort_sh, p.err));
-    tc_fence_after();
+  } else {
+    // ================================================================ epilogue
+    regs_increase<kRegsCompute>();
+    const int e = tid - 128;  // TMEM lane = query row of the tile
+    const uint32_t la = lane_base(warp);
+    bool ok = true;
+    int nq = 0;
+    // Q of an item: swizzled smem rows -> TMEM lanes (bf16 pairs), the A
+    // operand of S = Q K^T.
+    auto copy_q = [&](int buf) {
+      ok = ok && __all_sync(kFull, wait_bounded(&bars.q_full, nq & 1, &abort_sh, p.err));
+      ++nq;
+      if (ok) {
+        uint32_t r[D / 2];
+#pragma unroll
+        for (int ch = 0; ch < C::CHUNKS; ++ch)
+#pragma unroll
+          for (int pc = 0; pc < 8; ++pc) {
+            const uint4 v =
+                *reinterpret_cast<const uint4*>(sQ + ch * (BM * 128) + e * 128 + ((pc ^ (e & 7)) * 16));
+            r[ch * 32 + pc * 4 + 0] = v.x;
+            r[ch * 32 + pc * 4 + 1] = v.y;
+            r[ch * 32 + pc * 4 + 2] = v.z;
+            r[ch * 32 + pc * 4 + 3] = v.w;
+          }
+#pragma unroll
+        for (int q = 0; q < D / 64; ++q) {
+          uint32_t rr[32];
+#pragma unroll
+          for (int c = 0; c < 32; ++c) rr[c] = r[q * 32 + c];
+          tmem_st32(tmem + la + C::COL_Q + buf * 64 + q * 32, rr);
+        }
+        tmem_st_wait();
+      }
+      fence_proxy_async_smem();  // the next TMA write of sQ follows these reads
+      tc_fence_before();
+      mbar_arrive(&bars.qt_ready[buf]);
+      mbar_arrive(&bars.q_free);
+    };
+    ItemReader<DYN, true> items{(long long)blockIdx.x};
+    long long item = items.next(p, iq, &abort_sh);
+    if (item >= 0) copy_q(0);
+    for (int i = 0; item >= 0; ++i) {
+      const Work w = decode_work<MODE>(p, item);
+      const long long nxt = items.next(p, iq, &abort_sh);
+      if (nxt >= 0) copy_q((i + 1) & 1);
+      long long row, sample;
+      int head;
+      const bool row_ok = lane_row<MODE>(p, w, e, row, sample, head);
+      ok = ok && __all_sync(kFull, wait_bounded(&bars.l_ready[i & 1], (i >> 1) & 1, &abort_sh, p.err));
+      const float l_row = lfin[i & 1][e], m_row = mfin[i & 1][e];
+      mbar_arrive(&bars.l_free[i & 1]);
+      ok = ok && __all_sync(kFull, wait_bounded(&bars.o_full, i & 1, &abort_sh, p.err));
+      tc_fence_after();
+      float o[D];
+      tmem_ld_row<D>(tmem + la + C::COL_O, o);
+      tc_fence_before();
+      mbar_arrive(&bars.o_free);
+      const long long bh = (long long)w.b * p.Hq + head;
+      const float inv_l = (l_row > 0.f) ? 1.f / l_row : 0.f;
 
-    // ------------------------------------------------------------ epilogue
-    const long long bh = (long long)w.b * p.Hq + head;
-    const float inv_l = (l_run > 0.f) ? 1.f / l_run : 0.f;
-
-    if (EPI == EPI_BF16 || EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA || EPI == EPI_DELTA_BUILD) {
-      float* slot = reinterpret_cast<float*>(sK);  // K ring is idle once every MMA completed
-      const bool sampled = row_ok && is_sampled_row(row, p.gamma);
-      if (EPI == EPI_FUSED_INTILE) {
-        fence_proxy_async_smem();  // generic writes after the ring's TMA writes
-        // Pass 1: sampled rows publish their sparse output for the rows of their group.
-        float* dst = slot + (t / p.gamma) * D;
-#pragma unroll 1
-        for (int q = 0; q < D / 32; ++q) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_addr + C::COL_O + q * 32, r);
-          tmem_ld_wait();
+      if (EPI == EPI_BF16 || EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA || EPI == EPI_DELTA_BUILD) {
+#pragma unroll
+        for (int c = 0; c < D; ++c) o[c] *= inv_l;
+        const bool sampled = row_ok && is_sampled_row(row, p.gamma);
+        if (EPI == EPI_FUSED_INTILE) {
+          // Sampled rows publish their sparse output to the rows of their group.
+          named_bar_sync(2, 128);  // the previous item's readers are done with sbuf
           if (ok && sampled) {
+            float* dst = sbuf + (e / p.gamma) * D;
 #pragma unroll
-            for (int c = 0; c < 32; ++c) dst[q * 32 + c] = __uint_as_float(r[c]) * inv_l;
+            for (int c = 0; c < D; c += 4) *reinterpret_cast<float4*>(dst + c) = make_float4(o[c], o[c + 1], o[c + 2], o[c + 3]);
           }
+          named_bar_sync(2, 128);
         }
-        named_bar_sync(1, 128);
-      }
-#pragma unroll 1
-      for (int q = 0; q < D / 32; ++q) {
-        uint32_t r[32];
-        tmem_ld32(tmem + lane_addr + C::COL_O + q * 32, r);
-        tmem_ld_wait();
-        float v[32];
+        if (ok && row_ok) {
+          __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out_bf16) + (bh * p.N + row) * D;
 #pragma unroll
-        for (int c = 0; c < 32; ++c) v[c] = __uint_as_float(r[c]) * inv_l;
-        if (!ok || !row_ok) continue;
-        if (EPI == EPI_BF16) {
-          store_row_bf16<D>(reinterpret_cast<__nv_bfloat16*>(p.out_bf16) + (bh * p.N + row) * D + q * 32, v);
-          if (p.s_sampled != nullptr && sampled) store_f32x32(p.s_sampled + (bh * p.n_s + sample) * D + q * 32, v);
-        } else if (EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA) {
-          float dk[32];
-          load_f32x32(p.d_in + (bh * p.n_s + sample) * D + q * 32, dk);
-          if (!sampled) {
-            float corr[32];
-            if (EPI == EPI_FUSED_INTILE) {
-              const float* sk = slot + (t / p.gamma) * D + q * 32;
+          for (int q = 0; q < D / 32; ++q) {
+            float* v = o + q * 32;
+            if (EPI == EPI_BF16) {
+              store_bf16x32(orow + q * 32, v);
+              if (p.s_sampled != nullptr && sampled) store_f32x32(p.s_sampled + (bh * p.n_s + sample) * D + q * 32, v);
+            } else if (EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA) {
+              float dk[32];
+              load_f32x32(p.d_in + (bh * p.n_s + sample) * D + q * 32, dk);
+              if (!sampled) {
+                float corr[32];
+                if (EPI == EPI_FUSED_INTILE) {
+                  const float* sk = sbuf + (e / p.gamma) * D + q * 32;
 #pragma unroll
-              for (int c = 0; c < 32; ++c) corr[c] = dk[c] - sk[c];
-            } else {
-              load_f32x32(p.delta_in + (bh * p.n_s + sample) * D + q * 32, corr);
+                  for (int c = 0; c < 32; ++c) corr[c] = dk[c] - sk[c];
+                } else {
+                  load_f32x32(p.delta_in + (bh * p.n_s + sample) * D + q * 32, corr);
+                }
+#pragma unroll
+                for (int c = 0; c < 32; ++c) dk[c] = v[c] + corr[c];
+              }
+              store_bf16x32(orow + q * 32, dk);
+            } else {  // EPI_DELTA_BUILD: Delta_k = D_k - S_{k gamma}
+              float dk[32];
+              load_f32x32(p.d_in + (bh * p.n_s + sample) * D + q * 32, dk);
+#pragma unroll
+              for (int c = 0; c < 32; ++c) dk[c] -= v[c];
+              store_f32x32(p.delta_out + (bh * p.n_s + sample) * D + q * 32, dk);
             }
-#pragma unroll
-            for (int c = 0; c < 32; ++c) dk[c] = v[c] + corr[c];
           }
-          store_row_bf16<D>(reinterpret_cast<__nv_bfloat16*>(p.out_bf16) + (bh * p.N + row) * D + q * 32, dk);
-        } else {  // EPI_DELTA_BUILD: Delta_k = D_k - S_{k gamma}
-          float dk[32];
-          load_f32x32(p.d_in + (bh * p.n_s + sample) * D + q * 32, dk);
-#pragma unroll
-          for (int c = 0; c < 32; ++c) dk[c] -= v[c];
-          store_f32x32(p.delta_out + (bh * p.n_s + sample) * D + q * 32, dk);
-        }
-      }
-    } else {
-      // Dense sampled rows: the whole key range in this CTA, or split-K
-      // partials merged by the last CTA of the M-tile to finish.
-      const size_t slot_floats = (size_t)BM * (D + 2);
-      auto store_final = [&](int q, const float* v) {
-        if (EPI == EPI_DENSE_F32)
-          store_f32x32(p.d_out + (bh * p.n_s + sample) * D + q * 32, v);
-        else
-          store_row_bf16<D>(reinterpret_cast<__nv_bfloat16*>(p.out_bf16) + (bh * p.N + row) * D + q * 32, v);
-      };
-      if (w.n_chunks == 1) {
-#pragma unroll 1
-        for (int q = 0; q < D / 32; ++q) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_addr + C::COL_O + q * 32, r);
-          tmem_ld_wait();
-          float v[32];
-#pragma unroll
-          for (int c = 0; c < 32; ++c) v[c] = __uint_as_float(r[c]) * inv_l;
-          if (ok && row_ok) store_final(q, v);
         }
       } else {
-        float* part = p.partials + (size_t)w.unit * slot_floats;
-#pragma unroll 1
-        for (int q = 0; q < D / 32; ++q) {
-          uint32_t r[32];
-          tmem_ld32(tmem + lane_addr + C::COL_O + q * 32, r);
-          tmem_ld_wait();
-          float v[32];
+        // Dense sampled rows: the whole key range in this item, or split-K
+        // partials merged by the last CTA of the M-tile to finish.
+        const size_t slot_floats = (size_t)BM * (D + 2);
+        auto store_final = [&](int q, const float* v) {
+          if (EPI == EPI_DENSE_F32)
+            store_f32x32(p.d_out + (bh * p.n_s + sample) * D + q * 32, v);
+          else
+            store_bf16x32(reinterpret_cast<__nv_bfloat16*>(p.out_bf16) + (bh * p.N + row) * D + q * 32, v);
+        };
+        if (w.n_chunks == 1) {
+          if (ok && row_ok) {
 #pragma unroll
-          for (int c = 0; c < 32; ++c) v[c] = __uint_as_float(r[c]);
-          if (ok) store_f32x32(part + (size_t)t * D + q * 32, v);
-        }
-        if (ok) {
-          part[(size_t)BM * D + t] = m_run;
-          part[(size_t)BM * D + BM + t] = l_run;
-        }
-        __threadfence();
-        named_bar_sync(1, 128);
-        if (t == 0) {
-          const int prev = abort_sh ? -1 : atomicAdd(p.tickets + w.u0, 1);
-          ticket_sh = prev;
-          if (prev == w.n_chunks - 1) p.tickets[w.u0] = 0;  // ready for the next call
-        }
-        named_bar_sync(1, 128);
-        if (ticket_sh == w.n_chunks - 1 && row_ok) {
-          __threadfence();
-          float mstar = -INFINITY;
-          for (int c = 0; c < w.n_chunks; ++c)
-            mstar = fmaxf(mstar, __ldcg(p.partials + (size_t)(w.u0 + c) * slot_floats + (size_t)BM * D + t));
-          float lsum = 0.f;
-          for (int c = 0; c < w.n_chunks; ++c) {
-            const float* pc = p.partials + (size_t)(w.u0 + c) * slot_floats;
-            const float mc = __ldcg(pc + (size_t)BM * D + t);
-            if (mc != -INFINITY) lsum += __ldcg(pc + (size_t)BM * D + BM + t) * ex2(mc - mstar);
-          }
-          const float inv = (lsum > 0.f) ? 1.f / lsum : 0.f;
-#pragma unroll 1
-          for (int q = 0; q < D / 32; ++q) {
-            float v[32];
+            for (int q = 0; q < D / 32; ++q) {
+              float v[32];
 #pragma unroll
-            for (int c = 0; c < 32; ++c) v[c] = 0.f;
-            for (int c2 = 0; c2 < w.n_chunks; ++c2) {
-              const float* pc = p.partials + (size_t)(w.u0 + c2) * slot_floats;
-              const float mc = __ldcg(pc + (size_t)BM * D + t);
-              if (mc == -INFINITY) continue;
-              const float f = ex2(mc - mstar);
-              float o[32];
-              load_f32x32_cg(pc + (size_t)t * D + q * 32, o);
-#pragma unroll
-              for (int c = 0; c < 32; ++c) v[c] += o[c] * f;
+              for (int c = 0; c < 32; ++c) v[c] = o[q * 32 + c] * inv_l;
+              store_final(q, v);
             }
+          }
+        } else {
+          float* part = p.partials + (size_t)w.unit * slot_floats;
+          if (ok) {
 #pragma unroll
-            for (int c = 0; c < 32; ++c) v[c] *= inv;
-            store_final(q, v);
+            for (int q = 0; q < D / 32; ++q) store_f32x32(part + (size_t)e * D + q * 32, o + q * 32);
+            part[(size_t)BM * D + e] = m_row;
+            part[(size_t)BM * D + BM + e] = l_row;
+          }
+          __threadfence();
+          named_bar_sync(2, 128);
+          if (e == 0) {
+            const int prev = (ok && !abort_sh) ? atomicAdd(p.tickets + w.u0, 1) : -1;
+            ticket_sh = prev;
+            if (prev == w.n_chunks - 1) p.tickets[w.u0] = 0;  // ready for the next call
+          }
+          named_bar_sync(2, 128);
+          const bool merge = ticket_sh == w.n_chunks - 1;
+          named_bar_sync(2, 128);  // ticket_sh is rewritten by the next split item
+          if (merge && row_ok) {
+            __threadfence();
+            float mstar = -INFINITY;
+            for (int c = 0; c < w.n_chunks; ++c)
+              mstar = fmaxf(mstar, __ldcg(p.partials + (size_t)(w.u0 + c) * slot_floats + (size_t)BM * D + e));
+            float lsum = 0.f;
+            for (int c = 0; c < w.n_chunks; ++c) {
+              const float* pc = p.partials + (size_t)(w.u0 + c) * slot_floats;
+              const float mc = __ldcg(pc + (size_t)BM * D + e);
+              if (mc != -INFINITY) lsum += __ldcg(pc + (size_t)BM * D + BM + e) * ex2(mc - mstar);
+            }
+            const float inv = (lsum > 0.f) ? 1.f / lsum : 0.f;
+#pragma unroll 1
+            for (int q = 0; q < D / 32; ++q) {
+              float v[32];
+#pragma unroll
+              for (int c = 0; c < 32; ++c) v[c] = 0.f;
+              for (int c2 = 0; c2 < w.n_chunks; ++c2) {
+                const float* pc = p.partials + (size_t)(w.u0 + c2) * slot_floats;
+                const float mc = __ldcg(pc + (size_t)BM * D + e);
+                if (mc == -INFINITY) continue;
+                const float f = ex2(mc - mstar);
+                float x[32];
+                load_f32x32_cg(pc + (size_t)e * D + q * 32, x);
+#pragma unroll
+                for (int c = 0; c < 32; ++c) v[c] += x[c] * f;
+              }
+#pragma unroll
+              for (int c = 0; c < 32; ++c) v[c] *= inv;
+              store_final(q, v);
+            }
           }
         }
       }
+      item = nxt;
     }
   }
 

@@ -10,7 +10,11 @@ namespace da {
 
 template <int D, int MODE, int EPI>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
-                        long long grid, cudaStream_t s);
+                        long long n_items, cudaStream_t s);
+
+// Bytes of the epilogue buffer that holds the sampled sparse rows of one tile
+// when the Delta is fused inside the tile.
+constexpr unsigned kSampleBufBytes = 8192;
 
 unsigned attn_smem_bytes(int d);
 

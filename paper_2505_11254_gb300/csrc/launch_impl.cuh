@@ -5,14 +5,22 @@
 
 namespace da {
 
+// Persistent launch: min(items, SMs) CTAs, each walking items with a stride
+// of the grid size.
 template <int D, int MODE, int EPI>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
-                        long long grid, cudaStream_t s) {
+                        long long n_items, cudaStream_t s) {
   auto kfn = attn_kernel<D, MODE, EPI>;
   cudaError_t e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<D>::SMEM);
   if (e != cudaSuccess) return e;
-  if (grid <= 0) return cudaSuccess;
-  kfn<<<(unsigned)grid, kThreads, Cfg<D>::SMEM, s>>>(tq, tk, tv, p);
+  if (n_items <= 0) return cudaSuccess;
+  int dev = 0, sms = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  Params q = p;
+  q.n_items = n_items;
+  const long long grid = n_items < sms ? n_items : sms;
+  kfn<<<(unsigned)grid, kThreads, Cfg<D>::SMEM, s>>>(tq, tk, tv, q);
   return cudaGetLastError();
 }
 

@@ -50,6 +50,7 @@ struct Params {
   long long chunk;         // key tiles per unit
   long long n_units;       // units (= CTAs)
   long long n_multi;       // leading units that belong to split M-tiles
+  long long n_items;       // work items of the launched kernel
   // buffers
   void* out_bf16;          // [B,Hq,N,d] bf16
   float* s_sampled;        // [B,Hq,n_s,d] fp32, nullable
@@ -59,6 +60,7 @@ struct Params {
   float* delta_out;        // [B,Hq,n_s,d] fp32
   float* partials;         // n_multi slots of BM*(d+2) fp32
   int* tickets;            // n_multi
+  unsigned long long* counter;  // dynamic item counter (zeroed before the launch)
   int* err;                // device status word
 };
 

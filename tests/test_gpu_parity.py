@@ -30,6 +30,9 @@ CASES = [
     (1, 4, 4, 129, 64, 1, 1, 128),        # window = 1, gamma = 128
     (1, 2, 2, 1000, 128, 4, 256, 1000),   # a single sample
     (1, 4, 1, 1536, 128, 4, 300, 48),     # gamma 48 (not a divisor of 128), split-K
+    (1, 4, 2, 700, 128, 4, 100, 4),       # gamma 4 at d = 128: Delta built in a separate pass
+    (2, 2, 2, 300, 128, 2, 40, 2),        # gamma 2
+    (1, 4, 4, 520, 64, 4, 64, 4),         # gamma 4 at d = 64: fused in the tile
 ]
 
 
