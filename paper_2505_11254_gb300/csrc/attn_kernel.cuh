@@ -14,9 +14,12 @@
 //              then reads O out of TMEM, releases it, normalises, applies the
 //              Delta correction and writes the output.
 //   warp 8     TMA producer: Q of the next item, K/V tiles through a ring.
-//   warp 9     MMA issuer: S = Q K^T (Q from TMEM, K from smem) and
-//              O += P V (P from TMEM, V from smem); tcgen05.commit -> mbarriers.
-//   warps 10-11 idle (they complete the third warpgroup).
+//   warp 9     QK issuer: S = Q K^T (Q from TMEM, K from smem) once its K
+//              tile has landed and PV(g-2) has freed the S buffer.
+//   warp 10    PV issuer: O += P V (P from TMEM, V from smem) once the softmax
+//              has written P(g).  Two issuing threads keep the tensor pipe fed:
+//              neither waits on the other's inputs.
+//   warp 11    idle (it completes the third warpgroup).
 // Registers: launched at 168 per thread (384 x 168 = 64512); the third
 // warpgroup gives back to 72 and the softmax and epilogue warpgroups grow to
 // 216, so 2 x 128 x 216 + 128 x 72 = 64512 exactly.
@@ -67,9 +70,9 @@ struct Bars {
   uint64_t q_full, q_free;
   uint64_t qt_ready[2];
   uint64_t s_full[2], p_full[2];
-  uint64_t o_step, o_full, o_free;
+  uint64_t pv_done[2], o_full, o_free;
   uint64_t l_ready[2], l_free[2];
-  uint64_t drain;
+  uint64_t drain, drain2;
 };
 
 template <int N>
@@ -163,7 +166,7 @@ __device__ __forceinline__ void tmem_ld_row(uint32_t addr, float (&v)[NCOL]) {
 // items from a global counter, longest first, and publishes them to the other
 // roles through a small shared-memory queue; the others read them in order.
 constexpr int kQueue = 8;
-constexpr int kQueueReaders = 9;  // MMA thread + 4 softmax warps + 4 epilogue warps
+constexpr int kQueueReaders = 10;  // QK and PV threads + 4 softmax warps + 4 epilogue warps
 struct ItemQueue {
   long long item[kQueue];
   uint64_t full[kQueue], empty[kQueue];
@@ -235,10 +238,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars.l_ready[b], 128);
       mbar_init(&bars.l_free[b], 128);
     }
-    mbar_init(&bars.o_step, 1);
+    mbar_init(&bars.pv_done[0], 1);
+    mbar_init(&bars.pv_done[1], 1);
     mbar_init(&bars.o_full, 1);
     mbar_init(&bars.o_free, 128);
     mbar_init(&bars.drain, 1);
+    mbar_init(&bars.drain2, 1);
     for (int k = 0; k < kQueue; ++k) {
       mbar_init(&iq.full[k], 1);
       mbar_init(&iq.empty[k], kQueueReaders);
@@ -329,74 +334,81 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (nq > 0) wait_drain(&bars.q_full, (nq - 1) & 1, p.err);
     }
   } else if (warp == 9) {
-    // ================================================================ MMA issuer
+    // ================================================================ QK issuer
     regs_decrease<kRegsControl>();
     if ((tid & 31) == 0) {
-      const uint32_t ring_base = smem_u32(ring);
-      int c = 0;
+      // Shared-memory descriptor of ring slot 0; a slot or K-step adds its
+      // byte offset / 16 to the start-address field.
+      const uint64_t kdesc0 = sdesc_sw128(smem_u32(ring), 16, 1024);
       long long g = 0;
       bool ok = true;
-      struct Pend {
-        long long g;
-        int vslot, item_i;
-        uint32_t vph;
-        bool first, last;
-      } pend{0, 0, 0, 0, false, false};
-      bool has_pend = false;
-      auto issue_pv = [&](const Pend& pv) {
-        if (!wait_bounded(&bars.p_full[pv.g & 1], (pv.g >> 1) & 1, &abort_sh, p.err)) return false;
-        if (!wait_bounded(&bars.full[pv.vslot], pv.vph, &abort_sh, p.err)) return false;
-        if (pv.first && pv.item_i >= 1 && !wait_bounded(&bars.o_free, (pv.item_i - 1) & 1, &abort_sh, p.err))
-          return false;
-        tc_fence_after();
-        const uint32_t sb = tmem + C::COL_S + (uint32_t)(pv.g & 1) * BN;
-        const uint32_t vb = ring_base + pv.vslot * C::KV_BYTES;
-#pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk)
-          mma_ts(tmem + C::COL_O, sb + kk * 8, sdesc_sw128(vb + kk * 2048, BN * 128, 1024), C::IDESC_PV,
-                 (pv.first && kk == 0) ? 0u : 1u);
-        mma_commit(&bars.o_step);
-        mma_commit(&bars.empty[pv.vslot]);
-        if (pv.last) mma_commit(&bars.o_full);
-        return true;
-      };
       ItemReader<DYN, false> items{(long long)blockIdx.x};
       int i = 0;
       for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
         const Work w = decode_work<MODE>(p, item);
         if (!wait_bounded(&bars.qt_ready[i & 1], (i >> 1) & 1, &abort_sh, p.err)) { ok = false; break; }
-        tc_fence_after();
         const uint32_t qt = tmem + C::COL_Q + (uint32_t)(i & 1) * 64;
-        for (int j = 0; j < w.T; ++j) {
-          const int ks = c % NS;
-          const uint32_t kph = (c / NS) & 1;
-          ++c;
-          const int vs = c % NS;
-          const uint32_t vph = (c / NS) & 1;
-          ++c;
+        for (int j = 0; j < w.T; ++j, ++g) {
+          const int ks = (int)((2 * g) % NS);
+          const uint32_t kph = (uint32_t)((2 * g) / NS) & 1;
           if (!wait_bounded(&bars.full[ks], kph, &abort_sh, p.err)) { ok = false; break; }
+          // S buffer g&1 held P(g-2): PV(g-2) must have read it.
+          if (g >= 2 && !wait_bounded(&bars.pv_done[g & 1], (uint32_t)((g - 2) >> 1) & 1, &abort_sh, p.err)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
           const uint32_t sb = tmem + C::COL_S + (uint32_t)(g & 1) * BN;
-          const uint32_t kb = ring_base + ks * C::KV_BYTES;
+          const uint64_t kd = kdesc0 + ((ks * C::KV_BYTES) >> 4);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk)
-            mma_ts(sb, qt + kk * 8, sdesc_sw128(kb + (kk >> 2) * (BN * 128) + (kk & 3) * 32, 16, 1024),
-                   C::IDESC_QK, kk > 0 ? 1u : 0u);
+            mma_ts(sb, qt + kk * 8, kd + ((((kk >> 2) * (BN * 128)) + (kk & 3) * 32) >> 4), C::IDESC_QK,
+                   kk > 0 ? 1u : 0u);
           mma_commit(&bars.s_full[g & 1]);
-          mma_commit(&bars.empty[ks]);
-          if (has_pend && !issue_pv(pend)) { ok = false; break; }
-          pend = Pend{g, vs, i, vph, j == 0, j == w.T - 1};
-          has_pend = true;
-          ++g;
         }
       }
-      if (ok && has_pend) issue_pv(pend);
-      // Drain: all MMAs issued by this thread complete before TMEM is freed.
+      if (!ok)  // after an early exit, read the item queue to its end marker
+        while (items.next(p, iq, &abort_sh) >= 0) {}
       mma_commit(&bars.drain);
       wait_drain(&bars.drain, 0, p.err);
     }
-  } else if (warp >= 10) {
-    // idle warps of the control warpgroup
+  } else if (warp == 10) {
+    // ================================================================ PV issuer
+    regs_decrease<kRegsControl>();
+    if ((tid & 31) == 0) {
+      const uint64_t vdesc0 = sdesc_sw128(smem_u32(ring), BN * 128, 1024);
+      long long g = 0;
+      bool ok = true;
+      ItemReader<DYN, false> items{(long long)blockIdx.x};
+      int i = 0;
+      for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
+        const Work w = decode_work<MODE>(p, item);
+        for (int j = 0; j < w.T; ++j, ++g) {
+          const int vs = (int)((2 * g + 1) % NS);
+          const uint32_t vph = (uint32_t)((2 * g + 1) / NS) & 1;
+          if (!wait_bounded(&bars.p_full[g & 1], (g >> 1) & 1, &abort_sh, p.err)) { ok = false; break; }
+          if (!wait_bounded(&bars.full[vs], vph, &abort_sh, p.err)) { ok = false; break; }
+          // The epilogue must have read the previous item's O.
+          if (j == 0 && i >= 1 && !wait_bounded(&bars.o_free, (i - 1) & 1, &abort_sh, p.err)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t sb = tmem + C::COL_S + (uint32_t)(g & 1) * BN;
+          const uint64_t vd = vdesc0 + ((vs * C::KV_BYTES) >> 4);
+          mma_ts(tmem + C::COL_O, sb, vd, C::IDESC_PV, j == 0 ? 0u : 1u);
+#pragma unroll
+          for (int kk = 1; kk < BN / 16; ++kk)
+            mma_ts(tmem + C::COL_O, sb + kk * 8, vd + ((kk * 2048) >> 4), C::IDESC_PV, 1u);
+          mma_commit(&bars.pv_done[g & 1]);
+          mma_commit(&bars.empty[vs]);
+          if (j == w.T - 1) mma_commit(&bars.o_full);
+        }
+      }
+      if (!ok)
+        while (items.next(p, iq, &abort_sh) >= 0) {}
+      mma_commit(&bars.drain2);
+      wait_drain(&bars.drain2, 0, p.err);
+    }
+  } else if (warp == 11) {
+    // idle warp of the control warpgroup
     regs_decrease<kRegsControl>();
   } else if (warp < 4) {
     // ================================================================ softmax
@@ -420,6 +432,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
+        // S(g) landed, so QK(g) has read its K tile (ring position 2g).
+        if (t == 0) mbar_arrive(&bars.empty[(2 * g) % NS]);
         tc_fence_after();
         const uint32_t sb = C::COL_S + (uint32_t)(g & 1) * BN;
         float s[BN];
@@ -476,10 +490,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         f2_unpack(acc[2], a4, a5);
         f2_unpack(acc[3], a6, a7);
         const float l_tile = ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
-        // Rescale O (rare): PV(g-1) must have landed.  s_full(g) implies PV(g-2)
-        // completed, so the parity of PV(g-1) is unambiguous.
+        // Rescale O (rare): PV(g-1) must have landed.  QK(g) waited for PV(g-2),
+        // and PV(g+1) needs this thread's P(g+1), so the parity of PV(g-1) on
+        // its buffer is unambiguous.
         if (__any_sync(kFull, rescale)) {
-          if (!__all_sync(kFull, wait_bounded(&bars.o_step, (uint32_t)((g - 1) & 1), &abort_sh, p.err))) {
+          if (!__all_sync(kFull, wait_bounded(&bars.pv_done[(g - 1) & 1], (uint32_t)((g - 1) >> 1) & 1, &abort_sh, p.err))) {
             ok = false;
             break;
           }
@@ -529,7 +544,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Q of an item: swizzled smem rows -> TMEM lanes (bf16 pairs), the A
     // operand of S = Q K^T.
     auto copy_q = [&](int buf) {
-      ok = ok && __all_sync(kFull, wait_bounded(&bars.q_full, nq & 1, &abort_sh, p.err));
+      ok = ok && __all_sync(kFull, wait_sleepy(&bars.q_full, nq & 1, &abort_sh, p.err));
       ++nq;
       if (ok) {
         uint32_t r[D / 2];
@@ -568,10 +583,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       long long row, sample;
       int head;
       const bool row_ok = lane_row<MODE>(p, w, e, row, sample, head);
-      ok = ok && __all_sync(kFull, wait_bounded(&bars.l_ready[i & 1], (i >> 1) & 1, &abort_sh, p.err));
+      ok = ok && __all_sync(kFull, wait_sleepy(&bars.l_ready[i & 1], (i >> 1) & 1, &abort_sh, p.err));
       const float l_row = lfin[i & 1][e], m_row = mfin[i & 1][e];
       mbar_arrive(&bars.l_free[i & 1]);
-      ok = ok && __all_sync(kFull, wait_bounded(&bars.o_full, i & 1, &abort_sh, p.err));
+      ok = ok && __all_sync(kFull, wait_sleepy(&bars.o_full, i & 1, &abort_sh, p.err));
       tc_fence_after();
       float o[D];
       tmem_ld_row<D>(tmem + la + C::COL_O, o);

@@ -28,6 +28,23 @@ __device__ __forceinline__ bool wait_bounded(uint64_t* bar, uint32_t parity, vol
   }
 }
 
+// For waits that span a whole work item (the epilogue's): polls with a short
+// sleep so the waiting warp leaves the issue slots to the busy warps.
+__device__ __forceinline__ bool wait_sleepy(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
+    __nanosleep(200);
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
+      *abort_flag = 1;
+      atomicCAS(status, 0, kStatusTimeout);
+      return false;
+    }
+  }
+}
+
 // Used on the way out: waits for this CTA's own copies/MMAs even after an
 // abort, still with a time limit.
 __device__ __forceinline__ void wait_drain(uint64_t* bar, uint32_t parity, int* status) {
