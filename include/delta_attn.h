@@ -94,6 +94,22 @@ int strided_dense_workspace_size(int B, int Hq, int Hkv, int64_t N, int d, int g
 int strided_dense_attn(const void* Q, const void* K, const void* V, float* D_sampled, int B, int Hq, int Hkv,
                        int64_t N, int d, int gamma, void* workspace, size_t ws_bytes, void* stream);
 
+/* strided_dense_attn() for callers that cannot allocate device memory (their
+ * memory is owned by another allocator or budgeted up front, or their hot path
+ * must not allocate).  The paper has no counterpart: this is an integration
+ * variant.  Same arguments and results as strided_dense_attn() without the
+ * workspace: the split-K scratch lives in a fixed 16 MiB device array inside
+ * the library, held by every GPU that loads it until the process exits.  A
+ * shape whose scratch (strided_dense_workspace_size()) exceeds 16 MiB returns
+ * DA_ERR_WORKSPACE.  No call allocates: the first call on a device looks up
+ * the array's device address (so make that first call before any stream
+ * capture); every call then zeroes the scratch's tickets and counter on
+ * `stream` and launches the kernel.  All calls share the one array, so calls
+ * whose work overlaps on the GPU (different streams, or several host threads)
+ * race and must be serialised by the caller. */
+int strided_dense_attn_noalloc(const void* Q, const void* K, const void* V, float* D_sampled, int B, int Hq,
+                               int Hkv, int64_t N, int d, int gamma, void* stream);
+
 /* Eq. 6 as a separate pass: O_i = bf16(S_i + D_k - S_{k gamma}) for rows that
  * are not sampled and O_{k gamma} = bf16(D_k), with S_i read from the bf16
  * O_sparse and S_{k gamma} from S_sampled (fp32) or, when S_sampled is NULL,

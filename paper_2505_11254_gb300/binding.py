@@ -36,6 +36,7 @@ _SIGNATURES = {
     "sparse_window_attn": ([_p, _p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p], _i),
     "strided_dense_workspace_size": ([_i, _i, _i, _i64, _i, _i, ctypes.POINTER(_sz)], _i),
     "strided_dense_attn": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _p, _sz, _p], _i),
+    "strided_dense_attn_noalloc": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _p], _i),
     "delta_apply": ([_p, _p, _p, _p, _i, _i, _i64, _i, _i, _p], _i),
     "delta_attn_check": ([_p], _i),
     "delta_attn_status_string": ([_i], ctypes.c_char_p),
@@ -164,6 +165,17 @@ def strided_dense_attn(q, k, v, gamma, out=None, workspace=None, stream=None):
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check(load().strided_dense_attn(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, gamma,
                                      _dptr(workspace), ws_bytes, _stream(stream)), "strided_dense_attn")
+    return out
+
+
+def strided_dense_attn_noalloc(q, k, v, gamma, out=None, stream=None):
+    """strided_dense_attn without a workspace: the library's fixed device
+    scratch is used (for callers that cannot allocate)."""
+    B, Hq, Hkv, N, d = _qkv_shape(q, k, v)
+    if out is None:
+        out = torch.empty((B, Hq, n_samples(N, gamma), d), dtype=torch.float32, device=q.device)
+    _check(load().strided_dense_attn_noalloc(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, gamma,
+                                             _stream(stream)), "strided_dense_attn_noalloc")
     return out
 
 
