@@ -46,7 +46,11 @@ constexpr int kThreads = 384;
 constexpr int kRegsCompute = 216;  // softmax and epilogue warpgroups
 constexpr int kRegsControl = 72;   // producer / MMA warpgroup
 static_assert(2 * 128 * kRegsCompute + 128 * kRegsControl <= kThreads * 168, "register split above the launch total");
-constexpr float RESCALE_THRESHOLD = 8.0f;  // log2 units; O is rescaled only past this
+// O and the row sum are rescaled only when the running max grows by more than
+// this many log2 units.  Until then P = 2^(s - m) can reach 2^64: bf16 and fp32
+// share the 8-bit exponent, and 2^64 x 2^20 keys x |v| stays far below the
+// fp32 range, so the final O / l is unchanged (it is a ratio).
+constexpr float RESCALE_THRESHOLD = 64.0f;
 constexpr uint32_t kFull = 0xffffffffu;
 
 template <int D>
@@ -439,17 +443,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         float s[BN];
         tmem_ld_row<BN>(tmem + la + sb, s);
         if (tile_needs_mask<MODE>(p, w, j)) {
+          // Visible key offsets c of this tile: lo <= c <= hi (window and
+          // causality), plus c < se (sinks).  Branch-free selects; the sink
+          // term only in tiles that hold sink keys.
           const long long k0 = tile_index(w, j) * BN;
-          const int hi = (int)lmax(-1, lmin(BN - 1, row - k0));  // causal: key offset <= hi
-          int lo = 0, se = BN;                                    // band start, sink end
-          if (MODE != MODE_STRIDED_DENSE) {
-            lo = (int)lmax(0, lmin(BN, row - p.window + 1 - k0));
-            se = (int)lmax(0, lmin(BN, (long long)p.n_sink - k0));
-          }
+          const int hi = (int)lmax(-1, lmin(BN - 1, row - k0));
+          int lo = (MODE == MODE_STRIDED_DENSE) ? 0 : (int)lmax(0, lmin(BN, row - p.window + 1 - k0));
+          if (hi < lo) lo = BN + 1;  // empty range: (uint)(c - lo) is then above any width
+          const uint32_t width = hi >= lo ? (uint32_t)(hi - lo) : 0u;
+          if (MODE != MODE_STRIDED_DENSE && k0 < p.n_sink) {
+            const int se = (int)lmin(lmin(BN, (long long)p.n_sink - k0), (long long)hi + 1);
 #pragma unroll
-          for (int c = 0; c < BN; ++c) {
-            const bool vis = (c <= hi) && (c >= lo || c < se);
-            s[c] = vis ? s[c] : -INFINITY;
+            for (int c = 0; c < BN; ++c)
+              s[c] = ((uint32_t)(c - lo) <= width || c < se) ? s[c] : -INFINITY;
+          } else {
+#pragma unroll
+            for (int c = 0; c < BN; ++c) s[c] = ((uint32_t)(c - lo) <= width) ? s[c] : -INFINITY;
           }
         }
         float mx[4];
@@ -466,8 +475,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         float m_use = m_run;
         bool rescale = false;
         if (m_run == -INFINITY) {
-          m_use = mt;
-          rescale = (j > 0) && (mt != -INFINITY);  // O holds zeros; scaling by 0 keeps it so
+          m_use = mt;  // every earlier P of this row was 0, so O and l are exactly 0: nothing to rescale
         } else if (mt > m_run + RESCALE_THRESHOLD) {
           m_use = mt;
           rescale = true;
@@ -499,7 +507,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          const float f = !rescale ? 1.f : (m_run == -INFINITY) ? 0.f : ex2(m_run - m_use);
+          const float f = rescale ? ex2(m_run - m_use) : 1.f;
           l_run *= f;
 #pragma unroll
           for (int q = 0; q < D / 32; ++q) {
