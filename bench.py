@@ -35,6 +35,7 @@ if ROOT not in sys.path:
 import torch  # noqa: E402
 
 from paper_2505_11254_gb300 import flops  # noqa: E402
+from paper_2505_11254_gb300.replicas import Replicas  # noqa: E402
 from paper_2505_11254_gb300.inputs import WORKLOADS, LLAMA8B_N131K, generate, to_bits  # noqa: E402
 
 METRIC = "Δ-attn prefill tokens/s and useful TFLOP/s (% bf16 tensor peak) at N=131K/1M"
@@ -141,37 +142,6 @@ class ClockSampler:
                 "power_w_max": max(power) if power else None, "reasons": sorted(reasons), "samples": len(sm)}
 
 
-# ------------------------------------------------------------------ dist
-def dist_setup(n_gpus):
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    if world > 1:
-        import torch.distributed as dist
-        backend = "nccl" if torch.cuda.is_available() else "gloo"
-        if backend == "nccl":
-            torch.cuda.set_device(local)
-        dist.init_process_group(backend=backend)
-    elif torch.cuda.is_available():
-        torch.cuda.set_device(local)
-    return world, rank, local
-
-
-def barrier(world):
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
-
-
-def max_over_ranks(x, world):
-    if world == 1:
-        return x
-    import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
-
-
 # ------------------------------------------------------------------ oracle legs
 def oracle_sample(w, Qb, Kb, Vb, budget_s, max_groups=None):
     """Time the fp64 oracle on groups of gamma rows (all query heads) at evenly
@@ -217,9 +187,10 @@ def parity_spot_check(w, q, k, v, out, Qb, Kb, Vb):
 
 
 # ------------------------------------------------------------------ arms
-def run_reference(args, w, world, rank):
-    """Reference arm: the fp64 CPU oracle, each step a bounded sample."""
-    if rank != 0:
+def run_reference(args, w, rep):
+    """Reference arm: the fp64 CPU oracle, each step a bounded sample (rank 0
+    only; other ranks exit without work)."""
+    if rep.rank != 0:
         return
     q, k, v = generate(w, device="cpu")
     Qb, Kb, Vb = to_bits(q), to_bits(k), to_bits(v)
@@ -261,12 +232,13 @@ def config_of(w, n_gpus):
             "parallelism": "replicas: one independent sequence per GPU" if n_gpus > 1 else "single GPU"}
 
 
-def run_ours(args, w, world, rank, local):
+def run_ours(args, w, rep):
     from paper_2505_11254_gb300 import binding
+    world, rank, local = rep.world, rep.rank, rep.local
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
     peaks, peak_src = load_peaks()
-    wr = w.with_(seed=w.seed + rank)
+    wr = w.with_(seed=rep.seed(w.seed))
     q, k, v = generate(wr, device=dev)
     info = binding.plan_info(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, w.gamma)
     nk = int(info["kernels"])
@@ -295,7 +267,7 @@ def run_ours(args, w, world, rank, local):
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
-    barrier(world)
+    rep.barrier()
     torch.cuda.synchronize()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
@@ -304,16 +276,16 @@ def run_ours(args, w, world, rank, local):
         step(evs[s])
     t_end.record(stream)
     torch.cuda.synchronize()
-    barrier(world)
+    rep.barrier()
     clock_info = clocks.stop()
     status = binding.check()
     if status != binding.DA_OK:
         raise RuntimeError("device status %d after the timed loop" % status)
 
-    elapsed_ms = max_over_ranks(t_start.elapsed_time(t_end), world)
+    elapsed_ms = rep.max(t_start.elapsed_time(t_end))
     ms_per_step = elapsed_ms / args.steps
     tokens_per_step = w.B * w.N
-    value = world * tokens_per_step / (ms_per_step / 1e3)
+    value = rep.throughput(tokens_per_step, ms_per_step / 1e3)
 
     # per-kernel durations from the library's events (launching stream)
     names = (["strided_dense_f32", "sink_window_fused_delta"] if nk == 2 else
@@ -368,17 +340,17 @@ def run_ours(args, w, world, rank, local):
         for _ in range(max(1, args.warmup)):
             e2e_step()
         torch.cuda.synchronize()
-        barrier(world)
+        rep.barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(args.steps):
             e2e_step()
         e1.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = max_over_ranks(e0.elapsed_time(e1), world) / args.steps
+        e2e_ms = rep.max(e0.elapsed_time(e1)) / args.steps
         if binding.check() != binding.DA_OK:
             raise RuntimeError("device status after the e2e loop")
-        result["e2e"] = {"value": world * tokens_per_step / (e2e_ms / 1e3), "unit": UNIT,
+        result["e2e"] = {"value": rep.throughput(tokens_per_step, e2e_ms / 1e3), "unit": UNIT,
                          "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in (q, k, v)),
                          "d2h_bytes_per_step": out.numel() * out.element_size(), "ms_per_step": e2e_ms}
         del qh, kh, vh, oh, qd, kd, vd, od
@@ -424,16 +396,14 @@ def main():
         w = w.with_(window=args.window)
     if args.gamma is not None:
         w = w.with_(gamma=args.gamma)
-    world, rank, local = dist_setup(args.gpus)
+    rep = Replicas().init()
     try:
         if args.impl == "reference":
-            run_reference(args, w, world, rank)
+            run_reference(args, w, rep)
         else:
-            run_ours(args, w, world, rank, local)
+            run_ours(args, w, rep)
     finally:
-        if world > 1:
-            import torch.distributed as dist
-            dist.destroy_process_group()
+        rep.close()
 
 
 if __name__ == "__main__":
