@@ -77,6 +77,42 @@ int delta_attn_prefill_events(const void* Q, const void* K, const void* V, void*
                               int64_t N, int d, int n_sink, int64_t window, int gamma, void* workspace,
                               size_t ws_bytes, void* stream, void* const* events, int n_events);
 
+/* Output variants of delta_attn_prefill_ex(). */
+typedef enum {
+    DA_MODE_DELTA = 0,     /* Eq. 6: every row i gets Delta of sample floor(i/gamma)   */
+    DA_MODE_RECOMPUTE = 1  /* Eq. 5: only the sampled rows k*gamma become dense rows;
+                              every other row keeps its sink+window output            */
+} da_mode;
+
+/* Workspace bytes delta_attn_prefill_ex() needs for this shape, mode and dense
+ * tail (the sizes of delta_attn_workspace_size() plus the tail's split-K
+ * partials and tickets).  Writes *bytes; returns a da_status. */
+int delta_attn_workspace_size_ex(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma,
+                                 int mode, int64_t tail_dense, size_t* bytes);
+
+/* The prefill with the paper's two ablation forms.
+ *   mode: DA_MODE_DELTA (Eq. 6; the same result as delta_attn_prefill()) or
+ *         DA_MODE_RECOMPUTE (Eq. 5, the "recompute" form of Sec. 3: the
+ *         sink+window output for every row, the dense row at each sampled row
+ *         k*gamma, and no correction of the rows between samples).
+ *   tail_dense: 0 <= tail_dense <= N.  The last tail_dense rows
+ *         (N - tail_dense .. N - 1) are dense causal attention rows (appendix
+ *         "Implementation Details": a final block of queries recomputed
+ *         densely); the rows before it are unchanged by the tail.  The paper
+ *         does not give the block's size, so the caller chooses it; 0 means
+ *         no tail.
+ * Kernels, in stream order: the sampled-row and sparse passes of the chosen
+ * mode (Delta: strided dense, [strided sparse,] sink+window with the Delta
+ * epilogue; recompute: sink+window, then the dense sampled rows written over
+ * O), then, when tail_dense > 0, a dense pass over the tail rows written over
+ * O.  The sparse pass stops at the 128-row tile holding row N - tail_dense - 1.
+ * gamma = 1 ignores both options (every row is dense).  Layouts, workspace
+ * and error behaviour as delta_attn_prefill(); an unknown mode or a
+ * tail_dense outside [0, N] returns DA_ERR_INVALID_ARG. */
+int delta_attn_prefill_ex(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
+                          int d, int n_sink, int64_t window, int gamma, int mode, int64_t tail_dense,
+                          void* workspace, size_t ws_bytes, void* stream);
+
 /* f*(Q,K,V) of Alg. 1 alone: StreamingLLM sink + window attention of every
  * row, written as bf16 to O_sparse.  When S_sampled is not NULL the fp32
  * sparse rows at the sampled rows k*gamma are also written (the operand

@@ -21,6 +21,10 @@ DA_ERR_WORKSPACE = -4
 DA_ERR_CUDA = -5
 DA_ERR_TIMEOUT = -6
 
+DA_MODE_DELTA = 0
+DA_MODE_RECOMPUTE = 1
+_MODES = {"delta": DA_MODE_DELTA, "recompute": DA_MODE_RECOMPUTE}
+
 _lib = None
 
 _i = ctypes.c_int
@@ -31,6 +35,8 @@ _sz = ctypes.c_size_t
 _SIGNATURES = {
     "delta_attn_workspace_size": ([_i, _i, _i, _i64, _i, _i, _i64, _i, ctypes.POINTER(_sz)], _i),
     "delta_attn_prefill": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _sz, _p], _i),
+    "delta_attn_workspace_size_ex": ([_i, _i, _i, _i64, _i, _i, _i64, _i, _i, _i64, ctypes.POINTER(_sz)], _i),
+    "delta_attn_prefill_ex": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _i, _i64, _p, _sz, _p], _i),
     "delta_attn_prefill_events": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _sz, _p,
                                    ctypes.POINTER(_p), _i], _i),
     "sparse_window_attn": ([_p, _p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p], _i),
@@ -102,10 +108,14 @@ def _qkv_shape(q, k, v):
     return B, Hq, k.shape[1], N, d
 
 
-def workspace_size(B, Hq, Hkv, N, d, n_sink, window, gamma) -> int:
+def workspace_size(B, Hq, Hkv, N, d, n_sink, window, gamma, mode="delta", tail_dense=0) -> int:
     out = _sz(0)
-    _check(load().delta_attn_workspace_size(B, Hq, Hkv, N, d, n_sink, window, gamma, ctypes.byref(out)),
-           "delta_attn_workspace_size")
+    if mode == "delta" and tail_dense == 0:
+        _check(load().delta_attn_workspace_size(B, Hq, Hkv, N, d, n_sink, window, gamma, ctypes.byref(out)),
+               "delta_attn_workspace_size")
+    else:
+        _check(load().delta_attn_workspace_size_ex(B, Hq, Hkv, N, d, n_sink, window, gamma, _MODES[mode],
+                                                   tail_dense, ctypes.byref(out)), "delta_attn_workspace_size_ex")
     return out.value
 
 
@@ -120,14 +130,24 @@ def alloc_workspace(nbytes, device):
     return torch.empty(max(int(nbytes), 16), dtype=torch.uint8, device=device)
 
 
-def delta_attn_prefill(q, k, v, n_sink, window, gamma, out=None, workspace=None, stream=None):
-    """Delta Attention prefill (Alg. 1 / Eq. 6) -> bf16 [B,Hq,N,d]."""
+def delta_attn_prefill(q, k, v, n_sink, window, gamma, out=None, workspace=None, stream=None, mode="delta",
+                       tail_dense=0):
+    """Delta Attention prefill (Alg. 1 / Eq. 6) -> bf16 [B,Hq,N,d].
+
+    ``mode="recompute"`` gives the Eq. 5 form and ``tail_dense=t`` makes the
+    last t rows dense (both through delta_attn_prefill_ex)."""
     B, Hq, Hkv, N, d = _qkv_shape(q, k, v)
     if out is None:
         out = torch.empty_like(q)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
-    _check(load().delta_attn_prefill(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink, window,
-                                     gamma, _dptr(workspace), ws_bytes, _stream(stream)), "delta_attn_prefill")
+    if mode == "delta" and tail_dense == 0:
+        _check(load().delta_attn_prefill(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink,
+                                         window, gamma, _dptr(workspace), ws_bytes, _stream(stream)),
+               "delta_attn_prefill")
+    else:
+        _check(load().delta_attn_prefill_ex(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink,
+                                            window, gamma, _MODES[mode], tail_dense, _dptr(workspace), ws_bytes,
+                                            _stream(stream)), "delta_attn_prefill_ex")
     return out
 
 

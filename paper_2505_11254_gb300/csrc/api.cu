@@ -81,6 +81,11 @@ struct Plan {
   long long grid_sparse = 0, grid_dense = 0, grid_ssparse = 0;
   size_t off_d = 0, off_delta = 0, off_part = 0, off_ticket = 0, total = 0;
   size_t dense_part = 0, dense_ticket = 0, dense_total = 0;  // strided_dense_attn on its own
+  // Dense tail block: the rows N - tail .. N - 1 as dense causal attention,
+  // run as a strided-dense pass with gamma = 1 starting at row N - tail.
+  long long tail = 0;
+  Params pt;
+  size_t off_tail_part = 0, off_tail_ticket = 0;
 };
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -94,7 +99,31 @@ void packing(int G, int* Hp, int* R) {
   *R = BM / hp;
 }
 
-Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma, int sms) {
+// Split-K plan of a strided-dense pass over p.n_s samples: the chunk is chosen
+// so that about two units per SM exist; the longest M-tiles split, short ones
+// stay whole.
+void plan_split_k(Params& p, int sms) {
+  p.mtiles = cdiv(p.n_s, p.R);
+  long long total_tiles = 0;
+  for (long long t = 0; t < p.mtiles; ++t) total_tiles += strided_dense_len(p, t);
+  total_tiles *= (long long)p.B * p.groups_per_b;
+  p.chunk = std::max<long long>(8, cdiv(total_tiles, 2LL * std::max(sms, 1)));
+  long long units = 0, multi = 0;
+  for (long long t = 0; t < p.mtiles; ++t) {
+    long long nc = cdiv(strided_dense_len(p, t), p.chunk);
+    units += nc;
+    if (nc > 1) multi += nc;
+  }
+  p.n_units = units * p.B * p.groups_per_b;
+  p.n_multi = multi * p.B * p.groups_per_b;
+}
+
+// Bytes of the control block zeroed before a strided-dense launch: 4 item
+// counters, then one merge ticket per split unit.
+size_t ctrl_bytes(const Params& p) { return 4 * sizeof(unsigned long long) + (size_t)p.n_multi * sizeof(int); }
+
+Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma, int sms,
+               int64_t tail = 0) {
   Plan pl;
   Params& p = pl.p;
   p = Params{};
@@ -110,23 +139,10 @@ Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t win
   p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
   packing(p.G, &p.Hp, &p.R);
   p.groups_per_b = Hq / p.Hp;
-  p.mtiles = cdiv(p.n_s, p.R);
-  p.qtiles = cdiv(N, BM);
-
-  // Split-K: the chunk is chosen so that about two units per SM exist; the
-  // longest M-tiles split, short ones stay whole.
-  long long total_tiles = 0;
-  for (long long t = 0; t < p.mtiles; ++t) total_tiles += strided_dense_len(p, t);
-  total_tiles *= (long long)B * p.groups_per_b;
-  p.chunk = std::max<long long>(8, cdiv(total_tiles, 2LL * std::max(sms, 1)));
-  long long units = 0, multi = 0;
-  for (long long t = 0; t < p.mtiles; ++t) {
-    long long nc = cdiv(strided_dense_len(p, t), p.chunk);
-    units += nc;
-    if (nc > 1) multi += nc;
-  }
-  p.n_units = units * B * p.groups_per_b;
-  p.n_multi = multi * B * p.groups_per_b;
+  // Rows of the dense tail are recomputed densely afterwards, so the sparse
+  // pass stops at the q-tile holding row N - tail - 1.
+  p.qtiles = cdiv(N - tail, BM);
+  plan_split_k(p, sms);
 
   pl.grid_sparse = (long long)B * Hq * p.qtiles;
   pl.grid_dense = p.n_units;
@@ -135,8 +151,7 @@ Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t win
 
   const size_t rows_bytes = (size_t)B * Hq * p.n_s * d * sizeof(float);
   const size_t part_bytes = (size_t)p.n_multi * BM * (d + 2) * sizeof(float);
-  // control words zeroed before every call: 4 item counters, then the tickets
-  const size_t ticket_bytes = 4 * sizeof(unsigned long long) + (size_t)p.n_multi * sizeof(int);
+  const size_t ticket_bytes = ctrl_bytes(p);
   size_t off = 0;
   if (gamma >= 2) {
     pl.off_d = off;
@@ -150,6 +165,19 @@ Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t win
   off += align256(part_bytes);
   pl.off_ticket = off;
   off += align256(ticket_bytes);
+  if (tail > 0 && gamma >= 2) {
+    pl.tail = tail;
+    Params& t = pl.pt;
+    t = p;
+    t.gamma = 1;
+    t.n_s = tail;
+    t.row0 = N - tail;
+    plan_split_k(t, sms);
+    pl.off_tail_part = off;
+    off += align256((size_t)t.n_multi * BM * (d + 2) * sizeof(float));
+    pl.off_tail_ticket = off;
+    off += align256(ctrl_bytes(t));
+  }
   pl.total = off;
   pl.dense_part = 0;
   pl.dense_ticket = align256(part_bytes);
@@ -168,14 +196,19 @@ struct Maps {
   CUtensorMap q, qs, k, v;
 };
 
+// Sampled rows row0 + k * gamma of every (b, head): Hp heads x R samples a box.
+bool make_sample_map(CUtensorMap* m, const void* Q, const Params& p, int d) {
+  const long long row_bytes = (long long)d * 2;
+  const uint8_t* base = static_cast<const uint8_t*>(Q) + p.row0 * row_bytes;
+  return make_map(m, base, d, p.n_s, row_bytes * p.gamma, (long long)p.B * p.Hq, p.N * row_bytes, p.R, p.Hp);
+}
+
 bool make_maps(Maps* m, const void* Q, const void* K, const void* V, const Params& p, int d, bool need_rows,
                bool need_samples) {
   const long long row_bytes = (long long)d * 2;
   if (need_rows && !make_map(&m->q, Q, d, p.N, row_bytes, (long long)p.B * p.Hq, p.N * row_bytes, BM, 1))
     return false;
-  if (need_samples && !make_map(&m->qs, Q, d, p.n_s, row_bytes * p.gamma, (long long)p.B * p.Hq,
-                                p.N * row_bytes, p.R, p.Hp))
-    return false;
+  if (need_samples && !make_sample_map(&m->qs, Q, p, d)) return false;
   if (!make_map(&m->k, K, d, p.N, row_bytes, (long long)p.B * p.Hkv, p.N * row_bytes, BN, 1)) return false;
   if (!make_map(&m->v, V, d, p.N, row_bytes, (long long)p.B * p.Hkv, p.N * row_bytes, BN, 1)) return false;
   return true;
@@ -211,6 +244,20 @@ class ScopedWorkspace {
   bool owned_ = false, failed_ = false;
 };
 
+int check_variant(int mode, int64_t tail, int64_t N) {
+  if (mode != DA_MODE_DELTA && mode != DA_MODE_RECOMPUTE) return DA_ERR_INVALID_ARG;
+  if (tail < 0 || tail > N) return DA_ERR_INVALID_ARG;
+  return DA_OK;
+}
+
+// Kernel launches of one prefill call, in order.
+int prefill_kernels(const Plan& pl, int gamma, int mode) {
+  if (gamma == 1) return 1;
+  const int tail = pl.tail > 0 ? 1 : 0;
+  if (mode == DA_MODE_RECOMPUTE) return 2 + tail;
+  return (pl.fused_intile ? 2 : 3) + tail;
+}
+
 }  // namespace
 
 extern "C" {
@@ -236,6 +283,18 @@ int delta_attn_workspace_size(int B, int Hq, int Hkv, int64_t N, int d, int n_si
   int sms = 0;
   if ((rc = check_device(&sms))) return rc;
   *bytes = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms).total;
+  return DA_OK;
+}
+
+int delta_attn_workspace_size_ex(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma,
+                                 int mode, int64_t tail_dense, size_t* bytes) {
+  if (!bytes) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
+  if (rc) return rc;
+  if ((rc = check_variant(mode, tail_dense, N))) return rc;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  *bytes = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms, tail_dense).total;
   return DA_OK;
 }
 
@@ -271,17 +330,18 @@ int delta_attn_plan_info(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, i
 }
 
 static int prefill_impl(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
-                        int d, int n_sink, int64_t window, int gamma, void* workspace, size_t ws_bytes,
-                        void* stream, void* const* events, int n_events) {
+                        int d, int n_sink, int64_t window, int gamma, int mode, int64_t tail, void* workspace,
+                        size_t ws_bytes, void* stream, void* const* events, int n_events) {
   if (!Q || !K || !V || !O) return DA_ERR_INVALID_ARG;
   int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
   if (rc) return rc;
+  if ((rc = check_variant(mode, tail, N))) return rc;
   if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(workspace))
     return DA_ERR_MISALIGNED;
   int sms = 0;
   if ((rc = check_device(&sms))) return rc;
-  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms);
-  const int n_kernels = gamma == 1 ? 1 : (pl.fused_intile ? 2 : 3);
+  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms, tail);
+  const int n_kernels = prefill_kernels(pl, gamma, mode);
   if (n_events != 0 && (events == nullptr || n_events != n_kernels + 1)) return DA_ERR_INVALID_ARG;
   if (workspace != nullptr && ws_bytes < pl.total) return DA_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -289,6 +349,8 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   if ((rc = status_ptr(&p.err))) return rc;
   Maps m;
   if (!make_maps(&m, Q, K, V, p, d, gamma >= 2, true)) return DA_ERR_INVALID_ARG;
+  CUtensorMap q_tail;
+  if (pl.tail > 0 && !make_sample_map(&q_tail, Q, pl.pt, d)) return DA_ERR_INVALID_ARG;
 
   ScopedWorkspace ws(workspace, pl.total, s);
   if (ws.failed()) return DA_ERR_CUDA;
@@ -296,12 +358,27 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   p.partials = reinterpret_cast<float*>(base + pl.off_part);
   p.counter = reinterpret_cast<unsigned long long*>(base + pl.off_ticket);
   p.tickets = reinterpret_cast<int*>(base + pl.off_ticket + 4 * sizeof(unsigned long long));
-  if (cudaMemsetAsync(p.counter, 0, 4 * sizeof(unsigned long long) + p.n_multi * sizeof(int), s) != cudaSuccess)
-    return DA_ERR_CUDA;
+  if (cudaMemsetAsync(p.counter, 0, ctrl_bytes(p), s) != cudaSuccess) return DA_ERR_CUDA;
+  Params pt = pl.pt;
+  if (pl.tail > 0) {
+    pt.err = p.err;
+    pt.partials = reinterpret_cast<float*>(base + pl.off_tail_part);
+    pt.counter = reinterpret_cast<unsigned long long*>(base + pl.off_tail_ticket);
+    pt.tickets = reinterpret_cast<int*>(base + pl.off_tail_ticket + 4 * sizeof(unsigned long long));
+    pt.out_bf16 = O;
+    if (cudaMemsetAsync(pt.counter, 0, ctrl_bytes(pt), s) != cudaSuccess) return DA_ERR_CUDA;
+  }
 
   int ev = 0;
   auto mark = [&]() -> bool {
     return n_events == 0 || cudaEventRecord(static_cast<cudaEvent_t>(events[ev++]), s) == cudaSuccess;
+  };
+  // Appendix "Implementation Details": the final block of rows is replaced
+  // by dense rows, after every pass that writes rows of O.
+  auto run_tail = [&]() -> int {
+    if (pl.tail == 0) return DA_OK;
+    cudaError_t e = launch<MODE_STRIDED_DENSE, EPI_DENSE_BF16>(d, q_tail, m.k, m.v, pt, pt.n_units, s);
+    return (e == cudaSuccess && mark()) ? DA_OK : DA_ERR_CUDA;
   };
   if (!mark()) return DA_ERR_CUDA;
   cudaError_t e;
@@ -310,6 +387,16 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
     p.out_bf16 = O;
     e = launch<MODE_STRIDED_DENSE, EPI_DENSE_BF16>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
     return (e == cudaSuccess && mark()) ? DA_OK : DA_ERR_CUDA;
+  }
+  if (mode == DA_MODE_RECOMPUTE) {
+    // Eq. 5: sparse rows everywhere, then the sampled rows overwritten by
+    // their dense rows; no correction reaches the other rows.
+    p.out_bf16 = O;
+    e = launch<MODE_SPARSE, EPI_BF16>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+    if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
+    e = launch<MODE_STRIDED_DENSE, EPI_DENSE_BF16>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
+    if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
+    return run_tail();
   }
   float* dbuf = reinterpret_cast<float*>(base + pl.off_d);
   p.d_out = dbuf;
@@ -329,19 +416,29 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
     p.delta_in = delta;
     e = launch<MODE_SPARSE, EPI_FUSED_DELTA>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
   }
-  return (e == cudaSuccess && mark()) ? DA_OK : DA_ERR_CUDA;
+  if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
+  return run_tail();
 }
 
 int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
                        int d, int n_sink, int64_t window, int gamma, void* workspace, size_t ws_bytes,
                        void* stream) {
-  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, workspace, ws_bytes, stream, nullptr, 0);
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, DA_MODE_DELTA, 0, workspace, ws_bytes,
+                      stream, nullptr, 0);
+}
+
+int delta_attn_prefill_ex(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
+                          int d, int n_sink, int64_t window, int gamma, int mode, int64_t tail_dense,
+                          void* workspace, size_t ws_bytes, void* stream) {
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, mode, tail_dense, workspace, ws_bytes,
+                      stream, nullptr, 0);
 }
 
 int delta_attn_prefill_events(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv,
                               int64_t N, int d, int n_sink, int64_t window, int gamma, void* workspace,
                               size_t ws_bytes, void* stream, void* const* events, int n_events) {
-  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, workspace, ws_bytes, stream, events,
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, DA_MODE_DELTA, 0, workspace, ws_bytes,
+                      stream, events,
                       n_events);
 }
 

@@ -40,6 +40,7 @@ struct Params {
   long long window;
   int gamma;
   long long n_s;           // number of sampled rows ceil(N / gamma)
+  long long row0;          // row of sample 0: 0, or N - t for the dense tail block of t rows
   float scale_log2;        // log2(e) / sqrt(d)
   // sampled-row packing: Hp heads x R samples per tile (Hp * R == BM)
   int Hp, R;
@@ -99,7 +100,7 @@ __host__ __device__ __forceinline__ int sink_tiles_before(int n_sink, long long 
 // Number of key tiles an M-tile of sampled rows needs under causal masking.
 __host__ __device__ __forceinline__ long long strided_dense_len(const Params& p, long long t) {
   long long k_last = lmin(t * p.R + p.R - 1, p.n_s - 1);
-  return (k_last * p.gamma) / BN + 1;
+  return (p.row0 + k_last * p.gamma) / BN + 1;
 }
 
 // Split-K units are ordered longest-first: M-tile index t descending, then
@@ -203,7 +204,7 @@ __host__ __device__ __forceinline__ bool tile_needs_mask(const Params& p, const 
   if (MODE == MODE_SPARSE) {
     return !(k_end <= w.r0 && k_first > w.r_last - p.window);
   } else if (MODE == MODE_STRIDED_DENSE) {
-    return !(k_end <= w.r0 * p.gamma);
+    return !(k_end <= p.row0 + w.r0 * p.gamma);
   } else {
     return !(k_end <= w.r0 * p.gamma && k_first > w.r_last * p.gamma - p.window);
   }
@@ -221,7 +222,7 @@ __host__ __device__ __forceinline__ bool lane_row(const Params& p, const Work& w
   }
   head = w.h0 + t / p.R;
   sample = w.r0 + t % p.R;
-  row = sample * p.gamma;
+  row = p.row0 + sample * p.gamma;
   return sample < p.n_s;
 }
 

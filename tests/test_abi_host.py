@@ -82,3 +82,15 @@ def test_other_entry_points_reject_bad_arguments():
     sz = ctypes.c_size_t(0)
     assert lib.delta_attn_workspace_size(1, 2, 2, 64, 64, 0, 8, 0, ctypes.byref(sz)) == binding.DA_ERR_INVALID_ARG
     assert lib.delta_attn_workspace_size(1, 2, 2, 64, 64, 0, 8, 4, None) == binding.DA_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("mode,tail", [(2, 0), (-1, 0), (0, -1), (1, 257), (0, 1 << 40)])
+def test_prefill_ex_rejects_bad_mode_and_tail(mode, tail):
+    """Unknown output modes and dense tails outside [0, N] are rejected before
+    any device call (N = 256 here)."""
+    lib = binding.load()
+    assert lib.delta_attn_prefill_ex(_FAKE, _FAKE, _FAKE, _FAKE, 1, 4, 2, 256, 128, 4, 64, 16, mode, tail, None, 0,
+                                     None) == binding.DA_ERR_INVALID_ARG
+    sz = ctypes.c_size_t(0)
+    assert lib.delta_attn_workspace_size_ex(1, 4, 2, 256, 128, 4, 64, 16, mode, tail, ctypes.byref(sz)) == \
+        binding.DA_ERR_INVALID_ARG
