@@ -14,6 +14,8 @@ dense kernel, then the sink+window kernel with the fused Delta epilogue.
                  recorded by the library on the launching stream
   cpu_baseline   the fp64 oracle on the host cores over a bounded sample
   dense_baseline gamma = 1 through the same kernels (dense causal attention)
+  variants       the Eq. 5 "recompute" output and a dense tail block of --tail
+                 rows (appendix "Implementation Details"), timed the same way
 
 ``--impl reference`` times the oracle as the reference arm.  Multi-GPU: one
 process per GPU (torchrun), independent sequences per rank, no collective on
@@ -57,6 +59,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-dense-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-variants", action="store_true", help="skip the Eq. 5 / dense-tail timings")
+    ap.add_argument("--tail", type=int, default=1024, help="dense tail rows of the variant timings")
     return ap.parse_args()
 
 
@@ -232,6 +236,41 @@ def config_of(w, n_gpus):
             "parallelism": "replicas: one independent sequence per GPU" if n_gpus > 1 else "single GPU"}
 
 
+def time_variants(args, w, q, k, v, out, stream, restore):
+    """Median CUDA-event time of delta_attn_prefill_ex in the paper's ablation
+    forms: recompute (Eq. 5), Delta with a dense tail, recompute with a dense
+    tail.  The inputs are larger than L2, as in the main loop."""
+    from paper_2505_11254_gb300 import binding
+    res = {}
+    for name, mode, tail in (("recompute", "recompute", 0), ("delta_tail", "delta", args.tail),
+                             ("recompute_tail", "recompute", args.tail)):
+        ws = binding.alloc_workspace(binding.workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window,
+                                                            w.gamma, mode, tail), q.device)
+
+        def call():
+            binding.delta_attn_prefill(q, k, v, w.n_sink, w.window, w.gamma, out=out, workspace=ws, mode=mode,
+                                       tail_dense=tail)
+        for _ in range(3):
+            call()
+        torch.cuda.synchronize()
+        times = []
+        for _ in range(10):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            call()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+        if binding.check() != binding.DA_OK:
+            raise RuntimeError("device status after the %s timing" % name)
+        ms = statistics.median(times)
+        res[name] = {"mode": mode, "tail_dense": tail, "ms": ms, "tokens_per_s": w.B * w.N / (ms / 1e3),
+                     "tail_dense_pairs_per_head": flops.tail_pairs_per_head(w.N, tail)}
+        del ws
+    restore()  # `out` back to the Delta result for the spot check
+    return res
+
+
 def run_ours(args, w, rep):
     from paper_2505_11254_gb300 import binding
     world, rank, local = rep.world, rep.rank, rep.local
@@ -374,6 +413,9 @@ def run_ours(args, w, rep):
                                     "note": "gamma=1 through the same kernels = dense causal attention"}
         del dws
         step()  # restore `out` to the Delta result for the spot check
+
+    if not args.no_variants and rank == 0:
+        result["variants"] = time_variants(args, w, q, k, v, out, stream, step)
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         torch.cuda.synchronize()

@@ -40,6 +40,12 @@ def causal_pairs_per_head(N: int) -> int:
     return N * (N + 1) // 2
 
 
+def tail_pairs_per_head(N: int, tail: int) -> int:
+    """Dense rows N - tail .. N - 1 of the tail block: sum of (i + 1)."""
+    t = max(0, min(tail, N))
+    return causal_pairs_per_head(N) - causal_pairs_per_head(N - t)
+
+
 def useful_flops(B, Hq, N, d, n_sink, window, gamma) -> int:
     pairs = sparse_pairs_per_head(N, n_sink, window) + dense_pairs_per_head(N, gamma)
     return 4 * d * B * Hq * pairs

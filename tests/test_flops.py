@@ -55,3 +55,8 @@ def test_sampling_fraction():
 def test_dense_flops_gamma1():
     # gamma = 1 makes every row a dense causal row
     assert flops.dense_pairs_per_head(1000, 1) == flops.causal_pairs_per_head(1000)
+
+
+def test_tail_pairs_brute_force():
+    for N, t in ((1, 1), (10, 3), (300, 44), (517, 0), (64, 64), (64, 100)):
+        assert flops.tail_pairs_per_head(N, t) == sum(i + 1 for i in range(max(0, N - t), N))
