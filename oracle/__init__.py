@@ -8,7 +8,9 @@ Two independent statements of the method live here:
 * ``delta_oracle.c`` (wrapped below): direct per-row evaluation of Eq. 1
   (causal softmax attention), the StreamingLLM sink + window set, Eq. 4
   (sampled rows k*gamma), Alg. 1 / Eq. 6 (Delta correction), Eq. 5
-  ("recompute") and the appendix dense tail block, all in double precision.
+  ("recompute"), the appendix dense tail block and the appendix Delta
+  smoothing (linear interpolation, EMA, Alg. 2's alpha-beta-gamma filter),
+  all in double precision.
 * ``brute.py``: whole-matrix numpy evaluation (explicit N x N score matrix,
   -inf masks, matrix softmax, ``np.repeat`` of Delta) for small N.
 
@@ -44,6 +46,13 @@ def _load(path=None):
         lib.oracle_lemma1.argtypes = [u16p, u16p, u16p, ci, ci, ci, i64, ci, ci, i64, ci,
                                       ci, ci, i64, dp, dp, dp]
         lib.oracle_lemma1.restype = ci
+        lib.oracle_smooth_seq.argtypes = [ci, ctypes.c_double, ctypes.c_double, ctypes.c_double, dp, i64, ci, i64,
+                                          ci, i64, i64, dp]
+        lib.oracle_smooth_seq.restype = ci
+        lib.oracle_delta_attn_smoothed.argtypes = [u16p, u16p, u16p, ci, ci, ci, i64, ci, ci, i64, ci,
+                                                   ci, ci, ci, ci, i64, i64, ci, ctypes.c_double, ctypes.c_double,
+                                                   ctypes.c_double, i64, dp, dp, ci]
+        lib.oracle_delta_attn_smoothed.restype = ci
         _libs[path] = lib
     return _libs[path]
 
@@ -78,8 +87,27 @@ def bf16_bits_to_f64(a) -> np.ndarray:
     return (a.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
 
 
+SMOOTH_KINDS = {"none": 0, "linear": 1, "ema": 2, "abg": 3}
+
+
+def smooth_seq(kind, params, delta, n_s, gamma, rows, lib=None):
+    """Smoothed Delta corrections of rows [r0, r1) of one (batch, head)
+    (appendix "Interpolation"): ``delta`` [n_k, d] float64 holds Delta_0..;
+    ``params`` = (c1, c2, c3): EMA beta, or the filter's alpha, beta, gamma."""
+    delta = np.ascontiguousarray(delta, dtype=np.float64)
+    n_k, d = delta.shape
+    r0, r1 = rows
+    out = np.empty((r1 - r0, d), np.float64)
+    c1, c2, c3 = (tuple(params) + (0.0, 0.0, 0.0))[:3]
+    rc = _load(lib).oracle_smooth_seq(SMOOTH_KINDS[kind], c1, c2, c3, _ptr(delta, ctypes.c_double), n_k, d, n_s,
+                                      gamma, r0, r1, _ptr(out, ctypes.c_double))
+    if rc != 0:
+        raise ValueError("oracle_smooth_seq failed (invalid arguments)")
+    return out
+
+
 def delta_attn(Q, K, V, n_sink, window, gamma, *, batches=None, heads=None, rows=None,
-               mode="delta", tail_dense=0, nthreads=0, lib=None):
+               mode="delta", tail_dense=0, smooth="none", smooth_params=(), nthreads=0, lib=None):
     """Delta Attention (Alg. 1 / Eq. 6) over a box of batches, q-heads and rows.
 
     Returns a dict with float64 arrays ``A`` (corrected output A^V),
@@ -87,12 +115,28 @@ def delta_attn(Q, K, V, n_sink, window, gamma, *, batches=None, heads=None, rows
     the rows, first sample floor(r0/gamma)) and ``max_dev`` (max |sum p - 1|
     over every softmax vector evaluated).
     ``mode``: "delta" (Eq. 6) or "recompute" (Eq. 5).
+    ``smooth``: "none", "linear", "ema" or "abg" with ``smooth_params``
+    (appendix "Interpolation"; Eq. 6 mode only).  With smoothing only ``A``
+    and ``max_dev`` are returned.
     """
     Q, K, V = _u16(Q), _u16(K), _u16(V)
     B, Hq, Hkv, N, d = _shape(Q, K, V)
     b0, b1 = batches if batches is not None else (0, B)
     h0, h1 = heads if heads is not None else (0, Hq)
     r0, r1 = rows if rows is not None else (0, N)
+    if smooth != "none":
+        if mode != "delta":
+            raise ValueError("smoothing applies to the Eq. 6 output")
+        A = np.empty((b1 - b0, h1 - h0, r1 - r0, d), np.float64)
+        dev = ctypes.c_double(0.0)
+        c1, c2, c3 = (tuple(smooth_params) + (0.0, 0.0, 0.0))[:3]
+        rc = _load(lib).oracle_delta_attn_smoothed(
+            _ptr(Q, ctypes.c_uint16), _ptr(K, ctypes.c_uint16), _ptr(V, ctypes.c_uint16),
+            B, Hq, Hkv, N, d, n_sink, window, gamma, b0, b1, h0, h1, r0, r1,
+            SMOOTH_KINDS[smooth], c1, c2, c3, tail_dense, _ptr(A, ctypes.c_double), ctypes.byref(dev), nthreads)
+        if rc != 0:
+            raise ValueError("oracle_delta_attn_smoothed failed (invalid arguments)")
+        return {"A": A, "max_dev": dev.value}
     k0, k1 = r0 // gamma, (r1 - 1) // gamma + 1
     nb, nh, nr, nk = b1 - b0, h1 - h0, r1 - r0, k1 - k0
     S = np.empty((nb, nh, nr, d), np.float64)

@@ -16,7 +16,47 @@ def _masked_softmax(scores: np.ndarray, keep: np.ndarray) -> np.ndarray:
     return e / e.sum(axis=-1, keepdims=True)
 
 
-def delta_attn(Qf, Kf, Vf, n_sink, window, gamma, mode="delta", tail_dense=0):
+def smooth(kind, params, delta, N, gamma):
+    """Smoothed corrections for all N rows from the Delta rows [n_s, d]
+    (appendix "Interpolation"), each in a form unlike the C oracle's loop:
+    linear interpolation with ``np.interp`` through (k gamma, Delta_k), held
+    constant after the last sample; the EMA as one lower-triangular weight
+    matrix (row 0 keeps y_0, then weights beta (1-beta)^(i-j)); the
+    alpha-beta-gamma filter of Alg. 2 as the linear state-space recursion
+    x_k = M x_{k-1} + g Delta_k on the state (position, velocity,
+    acceleration) over the Delta rows, its outputs then repeated gamma times."""
+    n_s, d = delta.shape
+    y = np.repeat(delta, gamma, axis=0)[:N]
+    if kind == "none":
+        return y
+    if kind == "linear":
+        xs = np.arange(n_s) * gamma
+        rows = np.arange(N)
+        return np.stack([np.interp(rows, xs, delta[:, e]) for e in range(d)], axis=1)
+    if kind == "ema":
+        beta = params[0]
+        i = np.arange(N)[:, None]
+        j = np.arange(N)[None, :]
+        W = np.where(j <= i, beta * (1.0 - beta) ** np.maximum(i - j, 0), 0.0)
+        W[:, 0] = (1.0 - beta) ** np.arange(N)
+        return W @ y
+    al, be, ga = params
+    # predict p+v+a/2, v+a; residual r = y - predicted p; p += al r, v += be r, a += ga r
+    M = np.array([[1.0 - al, 1.0 - al, 0.5 * (1.0 - al)],
+                  [-be, 1.0 - be, 1.0 - 0.5 * be],
+                  [-ga, -ga, 1.0 - 0.5 * ga]])
+    g = np.array([al, be, ga])
+    out = np.empty_like(delta)
+    x = np.stack([delta[0], np.zeros(d), np.zeros(d)])     # [3, d]
+    out[0] = delta[0]
+    for k in range(1, n_s):
+        x = M @ x + np.outer(g, delta[k])
+        out[k] = x[0]
+    return np.repeat(out, gamma, axis=0)[:N]
+
+
+def delta_attn(Qf, Kf, Vf, n_sink, window, gamma, mode="delta", tail_dense=0, smooth_kind="none",
+               smooth_params=()):
     """Qf [B,Hq,N,d], Kf/Vf [B,Hkv,N,d] float64.  Returns (A_hat, S, D_full).
 
     Eq. 1 attention matrix sigma(QK^T/sqrt(d)) with the causal mask; the
@@ -43,7 +83,7 @@ def delta_attn(Qf, Kf, Vf, n_sink, window, gamma, mode="delta", tail_dense=0):
             AsV = _masked_softmax(scores, sparse) @ Vh       # sparse attention, every row
             delta = AV[::gamma] - AsV[::gamma]               # rows i with i mod gamma == 0
             if mode == "delta":
-                corr = np.repeat(delta, gamma, axis=0)[:N]
+                corr = smooth(smooth_kind, smooth_params, delta, N, gamma)
             else:                                            # Eq. 5: only the sampled rows move
                 corr = np.zeros_like(AsV)
                 corr[::gamma] = delta

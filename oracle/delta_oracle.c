@@ -26,6 +26,9 @@
  *     unchanged.
  *   - Appendix "Restatement and proof of Lemma 1": the error bound, evaluated
  *     here for the actual selected set W(i) (the proof holds for any set).
+ *   - Appendix "Interpolation" and Alg. 2: smoothing of the Delta corrections
+ *     (linear interpolation, EMA, alpha-beta-gamma filter) before they are
+ *     added to the sparse rows.
  *
  * Readings of the paper used here (each also listed in the design notes):
  *   - Rows are 0-based and the sample for row i is row floor(i/gamma)*gamma,
@@ -503,4 +506,172 @@ int oracle_lemma1(const uint16_t *Q, const uint16_t *K, const uint16_t *V,
     if (h_frac) *h_frac = H / (H + T);
     free(e); free(dense); free(sparse); free(head); free(vmax);
     return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Delta smoothing (appendix "Interpolation", Alg. 2).                       */
+/*                                                                          */
+/* With y_i = Delta_{floor(i/gamma)} (Alg. 1's repeat: one vector per row),  */
+/* the correction added to row i becomes                                    */
+/*   SMOOTH_LINEAR: (1 - b_i) Delta_k + b_i Delta_{k+1}, k = floor(i/gamma),  */
+/*       b_i = (i - k gamma) / gamma, rising linearly from 0 at the sample    */
+/*       towards 1 at the next one; the last group has no next sample and     */
+/*       keeps Delta_k;                                                       */
+/*   SMOOTH_EMA (c1 = beta): over the expanded rows, e_0 = y_0 and            */
+/*       e_i = (1 - beta) e_{i-1} + beta y_i;                                 */
+/*   SMOOTH_ABG (c1, c2, c3 = the filter's alpha, beta, gamma): Alg. 2 run    */
+/*       over the Delta vectors themselves (its output has one vector per    */
+/*       Delta), elementwise: position p = Delta_0, velocity v = 0,           */
+/*       acceleration a = 0, output Delta_0 for sample 0; at each later       */
+/*       sample predict p + v + a/2 and v + a, take the residual r = Delta_k  */
+/*       minus the predicted position, correct p, v and a by alpha r, beta r  */
+/*       and gamma r, and output p; row i then takes the output of its sample */
+/*       floor(i/gamma), as in Alg. 1's repeat.                               */
+/* SMOOTH_NONE gives y_i itself (Eq. 6).                                     */
+
+#define SMOOTH_NONE 0
+#define SMOOTH_LINEAR 1
+#define SMOOTH_EMA 2
+#define SMOOTH_ABG 3
+
+/*
+ * oracle_smooth_seq — the smoothed corrections of rows [r0, r1) of one
+ * (batch, head), computed by running the recurrence from row 0.
+ *   delta [n_k, d]: Delta_0 .. Delta_{n_k - 1}; n_k must reach the last sample
+ *         the rows use (one more for SMOOTH_LINEAR, unless it is the last of
+ *         the n_s samples).
+ *   corr  [r1 - r0, d].
+ * Returns 0, or -1 on invalid arguments.
+ */
+int oracle_smooth_seq(int kind, double c1, double c2, double c3,
+                      const double *delta, int64_t n_k, int d, int64_t n_s, int gamma,
+                      int64_t r0, int64_t r1, double *corr)
+{
+    if (!delta || !corr || d < 1 || gamma < 1 || n_s < 1 || r0 < 0 || r1 <= r0) return -1;
+    if (kind < SMOOTH_NONE || kind > SMOOTH_ABG) return -1;
+    int64_t last = (r1 - 1) / gamma;                 /* last sample used */
+    if (last >= n_s) return -1;
+    if (kind == SMOOTH_LINEAR && last + 1 < n_s) last += 1;
+    if (n_k <= last) return -1;
+
+    double *filt = NULL;                             /* Alg. 2 output per sample */
+    if (kind == SMOOTH_ABG) {
+        filt = (double *)malloc(sizeof(double) * (size_t)((last + 1) * d));
+        if (!filt) return -1;
+        for (int e = 0; e < d; ++e) {
+            double p = delta[e], v = 0.0, a = 0.0;
+            filt[e] = p;
+            for (int64_t k = 1; k <= last; ++k) {
+                const double p_pred = p + v + 0.5 * a;
+                const double v_pred = v + a;
+                const double r = delta[k * d + e] - p_pred;
+                p = p_pred + c1 * r;
+                v = v_pred + (MUTANT(10) ? c1 : c2) * r;
+                a = a + c3 * r;
+                filt[k * d + e] = p;
+            }
+        }
+    }
+    for (int e = 0; e < d; ++e) {
+        double ema = delta[e];                       /* EMA state */
+        for (int64_t i = 0; i < r1; ++i) {
+            const int64_t k = i / gamma;
+            const double y = delta[k * d + e];
+            double out;
+            if (kind == SMOOTH_NONE) {
+                out = y;
+            } else if (kind == SMOOTH_LINEAR) {
+                const double b = (double)(i - k * gamma + MUTANT(11)) / (double)gamma;
+                const double next = (k + 1 < n_s) ? delta[(k + 1) * d + e] : y;
+                out = (1.0 - b) * y + b * next;
+            } else if (kind == SMOOTH_EMA) {
+                if (i > 0)
+                    ema = MUTANT(9) ? c1 * ema + (1.0 - c1) * y : (1.0 - c1) * ema + c1 * y;
+                out = ema;
+            } else {
+                out = filt[k * d + e];
+            }
+            if (i >= r0) corr[(i - r0) * d + e] = out;
+        }
+    }
+    free(filt);
+    return 0;
+}
+
+typedef struct {
+    const problem *p;
+    int b0, h0, nh;
+    int64_t nk;              /* samples 0..nk-1 per (b, h) */
+    double *delta;           /* [nbh, nk, d] */
+} smooth_delta_ctx;
+
+static void smooth_delta_item(void *vc, int64_t it, double *prob, double *dev)
+{
+    /* Delta_k = (dense row k gamma) - (sparse row k gamma), Alg. 1 */
+    smooth_delta_ctx *c = (smooth_delta_ctx *)vc;
+    const problem *p = c->p;
+    const int d = p->d;
+    int64_t k = it % c->nk, bh = it / c->nk;
+    int b = c->b0 + (int)(bh / c->nh), h = c->h0 + (int)(bh % c->nh);
+    double *dst = c->delta + it * d;
+    double *sp = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!sp) return;
+    double e = attn_row(p, b, h, k * p->gamma, SET_CAUSAL, dst, prob);
+    if (e > *dev) *dev = e;
+    e = attn_row(p, b, h, k * p->gamma, SET_SPARSE, sp, prob);
+    if (e > *dev) *dev = e;
+    for (int x = 0; x < d; ++x) dst[x] -= sp[x];
+    free(sp);
+}
+
+/*
+ * oracle_delta_attn_smoothed — Eq. 6 with smoothed corrections over a box of
+ * batches [b0,b1), q-heads [h0,h1) and rows [r0,r1):
+ *   A_out[b, h, i] = S_i + corr_i (corr from oracle_smooth_seq), and rows
+ *   i >= N - tail_dense replaced by their dense rows.
+ * Returns 0, or -1 on invalid arguments / allocation failure.
+ */
+int oracle_delta_attn_smoothed(const uint16_t *Q, const uint16_t *K, const uint16_t *V,
+                               int B, int Hq, int Hkv, int64_t N, int d,
+                               int n_sink, int64_t window, int gamma,
+                               int b0, int b1, int h0, int h1, int64_t r0, int64_t r1,
+                               int kind, double c1, double c2, double c3, int64_t tail_dense,
+                               double *A_out, double *max_dev, int nthreads)
+{
+    problem p = {Q, K, V, B, Hq, Hkv, d, n_sink, gamma, N, window};
+    if (!valid_problem(&p) || !A_out) return -1;
+    if (b0 < 0 || b1 > B || b0 >= b1 || h0 < 0 || h1 > Hq || h0 >= h1) return -1;
+    if (r0 < 0 || r1 > N || r0 >= r1 || tail_dense < 0) return -1;
+    if (kind < SMOOTH_NONE || kind > SMOOTH_ABG) return -1;
+    const int64_t n_s = (N + gamma - 1) / gamma;
+    int64_t nk = (r1 - 1) / gamma + 1;
+    if (kind == SMOOTH_LINEAR && nk < n_s) nk += 1;
+    const int nh = h1 - h0;
+    const int64_t nbh = (int64_t)(b1 - b0) * nh, nr = r1 - r0;
+
+    double *delta = (double *)malloc(sizeof(double) * (size_t)(nbh * nk * d));
+    double *S = (double *)malloc(sizeof(double) * (size_t)(nbh * nr * d));
+    double *corr = (double *)malloc(sizeof(double) * (size_t)(nr * d));
+    int rc = (delta && S && corr) ? 0 : -1;
+    double dev = 0.0;
+    if (rc == 0) {
+        smooth_delta_ctx dc = {&p, b0, h0, nh, nk, delta};
+        rc |= run_pool(smooth_delta_item, &dc, nbh * nk, N, d, nthreads, &dev);
+        box_ctx sc;
+        memset(&sc, 0, sizeof sc);
+        sc.p = &p; sc.b0 = b0; sc.b1 = b1; sc.h0 = h0; sc.h1 = h1; sc.r0 = r0; sc.r1 = r1;
+        sc.S = S; sc.A = A_out; sc.tail_dense = tail_dense;
+        rc |= run_pool(box_sparse_item, &sc, nbh * nr, N, d, nthreads, &dev);
+        for (int64_t bh = 0; rc == 0 && bh < nbh; ++bh) {
+            rc |= oracle_smooth_seq(kind, c1, c2, c3, delta + bh * nk * d, nk, d, n_s, gamma, r0, r1, corr);
+            for (int64_t x = 0; x < nr * d; ++x) A_out[bh * nr * d + x] = S[bh * nr * d + x] + corr[x];
+        }
+        if (rc == 0 && tail_dense > 0)
+            rc |= run_pool(box_tail_item, &sc, nbh * nr, N, d, nthreads, &dev);
+    }
+    if (max_dev) *max_dev = dev;
+    free(delta);
+    free(S);
+    free(corr);
+    return rc;
 }

@@ -17,6 +17,14 @@ What pins what:
   * GQA head mapping         -> explicit repetition of the KV heads.
   * Lemma 1                  -> the appendix inequality on every sample.
   * whole-matrix restatement -> the numpy brute force (oracle/brute.py).
+  * Delta smoothing          -> reductions to Eq. 6 (EMA beta = 1, filter
+    (appendix Interpolation,    (1, 0, 0), linear at gamma = 1), fixed points
+     Alg. 2)                    of a constant Delta, the EMA step response,
+                                exactness of linear interpolation on affine
+                                Delta sequences, the filter's transfer function
+                                (impulse response summed against w^k) and its
+                                steady-state lag 6 (alpha - 1) / gamma on a
+                                cubic input (final-value theorem).
 """
 import numpy as np
 import torch
@@ -239,9 +247,102 @@ def pin_rows_agree(lib=None):
         assert np.abs(r["D_sample"][t] - full["D"][b, h, i // 9]).max() <= TOL
 
 
+def pin_smooth_reductions(lib=None):
+    """Smoothing forms that reduce to plain Eq. 6 or to each other: EMA with
+    beta = 1 and the filter with (1, 0, 0) give the repeated Delta; at gamma = 1
+    linear interpolation gives Delta itself and the filter with (alpha, 0, 0)
+    is the EMA with beta = alpha; a constant Delta is a fixed point of every
+    form; the box evaluation with smoothing "none" is the Eq. 6 box."""
+    rng = np.random.default_rng(7)
+    n_s, g, N, d = 9, 5, 43, 4
+    delta = rng.standard_normal((n_s, d))
+    plain = np.repeat(delta, g, axis=0)[:N]
+    for kind, par in (("ema", (1.0,)), ("abg", (1.0, 0.0, 0.0)), ("none", ())):
+        assert np.abs(oracle.smooth_seq(kind, par, delta, n_s, g, (0, N), lib=lib) - plain).max() <= TOL, kind
+    assert np.abs(oracle.smooth_seq("linear", (), delta, n_s, 1, (0, n_s), lib=lib) - delta).max() <= TOL
+    a = oracle.smooth_seq("abg", (0.3, 0.0, 0.0), delta, n_s, 1, (0, n_s), lib=lib)
+    b = oracle.smooth_seq("ema", (0.3,), delta, n_s, 1, (0, n_s), lib=lib)
+    assert np.abs(a - b).max() <= TOL
+    const = np.tile(rng.standard_normal((1, d)), (n_s, 1))
+    for kind, par in (("linear", ()), ("ema", (0.37,)), ("abg", (0.2, 0.05, 0.0035)), ("abg", (0.5, 0.4, 0.1))):
+        out = oracle.smooth_seq(kind, par, const, n_s, g, (3, N), lib=lib)
+        assert np.abs(out - const[0]).max() <= 1e-12, kind
+    Q, K, V = rand_bits(40, (1, 2, 45, 8)), rand_bits(41, (1, 1, 45, 8)), rand_bits(42, (1, 1, 45, 8))
+    ref = oracle.delta_attn(Q, K, V, 2, 6, 4, lib=lib)["A"]
+    got = oracle.delta_attn(Q, K, V, 2, 6, 4, smooth="ema", smooth_params=(1.0,), lib=lib)["A"]
+    assert np.abs(got - ref).max() <= TOL
+
+
+def _abg_transfer(al, be, ga, w):
+    """Transfer function from the filter input to its position output at
+    z^-1 = w, from the state-space form of Alg. 2 (x_k = M x_{k-1} + g y_k):
+    (2a + (2b + c - 4a) w + (2a - 2b + c) w^2) /
+    (2 + (2a + 2b + c - 6) w + (6 - 4a - 2b + c) w^2 + (2a - 2) w^3)."""
+    num = 2 * al + (2 * be + ga - 4 * al) * w + (2 * al - 2 * be + ga) * w ** 2
+    den = 2 + (2 * al + 2 * be + ga - 6) * w + (6 - 4 * al - 2 * be + ga) * w ** 2 + (2 * al - 2) * w ** 3
+    return num / den
+
+
+def pin_smooth_closed_forms(lib=None):
+    """EMA step response 1 - (1 - beta)^(i - gamma + 1); linear interpolation
+    exact on an affine Delta sequence (held after the last sample); the
+    filter's impulse response summed against w^k equals w H(w); the filter
+    tracks a cubic with the constant lag 6 (alpha - 1) / gamma."""
+    g, n_s, beta = 4, 10, 0.3
+    step = np.zeros((n_s, 1))
+    step[1:] = 1.0
+    e = oracle.smooth_seq("ema", (beta,), step, n_s, g, (0, n_s * g), lib=lib)[:, 0]
+    i = np.arange(n_s * g)
+    want = np.where(i < g, 0.0, 1.0 - (1.0 - beta) ** np.maximum(i - g + 1, 0))
+    assert np.abs(e - want).max() <= TOL
+    aff = (0.25 + 0.5 * np.arange(n_s))[:, None] * np.array([[1.0, -2.0]])
+    lin = oracle.smooth_seq("linear", (), aff, n_s, g, (0, n_s * g), lib=lib)
+    want = (0.25 + 0.5 * np.minimum(i / g, n_s - 1))[:, None] * np.array([[1.0, -2.0]])
+    assert np.abs(lin - want).max() <= TOL
+    for (al, be, ga) in ((0.2, 0.05, 0.0035), (0.5, 0.4, 0.1), (0.1, 5e-3, 1.66e-4)):
+        n = 400
+        imp = np.zeros((n, 1))
+        imp[1] = 1.0
+        o = oracle.smooth_seq("abg", (al, be, ga), imp, n, 1, (0, n), lib=lib)[:, 0]
+        w = 0.5
+        assert abs(np.sum(o * w ** np.arange(n)) - w * _abg_transfer(al, be, ga, w)) <= 1e-12, (al, be, ga)
+    al, be, ga = 0.2, 0.05, 0.0035
+    n = 3000
+    cubic = (np.arange(n, dtype=np.float64) ** 3 * 1e-6)[:, None]
+    o = oracle.smooth_seq("abg", (al, be, ga), cubic, n, 1, (0, n), lib=lib)[:, 0]
+    lag = o[-1] - cubic[-1, 0]
+    assert abs(lag - 6e-6 * (al - 1) / ga) <= 1e-6 * abs(lag), lag
+
+
+def pin_smooth_brute(lib=None):
+    """The smoothed prefill (direct per-row evaluation) equals the whole-matrix
+    numpy restatement with its own smoothing forms, over gamma, window, GQA,
+    the three forms and the dense tail."""
+    seed = 500
+    for idx, (gamma, window, kind, par) in enumerate((
+            (4, 7, "linear", ()), (3, 16, "ema", (0.5,)), (5, 2, "abg", (0.2, 0.05, 0.0035)),
+            (1, 5, "ema", (0.75,)), (16, 9, "linear", ()), (7, 64, "abg", (0.1, 5e-3, 1.66e-4)))):
+        seed += 3
+        Hkv, G = 1 + idx % 2, (1, 2, 4)[idx % 3]
+        N, d = (61, 40, 53)[idx % 3], 8
+        Q, K, V = rand_bits(seed, (1, Hkv * G, N, d), 1.5), rand_bits(seed + 1, (1, Hkv, N, d), 1.5), \
+            rand_bits(seed + 2, (1, Hkv, N, d))
+        tail = 6 if idx % 2 else 0
+        A_b, _, _ = brute.delta_attn(f64(Q), f64(K), f64(V), 2, window, gamma, tail_dense=tail, smooth_kind=kind,
+                                     smooth_params=par)
+        got = oracle.delta_attn(Q, K, V, 2, window, gamma, tail_dense=tail, smooth=kind, smooth_params=par,
+                                lib=lib)["A"]
+        assert np.abs(got - A_b).max() <= TOL, (gamma, window, kind)
+        r0 = N // 3
+        part = oracle.delta_attn(Q, K, V, 2, window, gamma, rows=(r0, N), tail_dense=tail, smooth=kind,
+                                 smooth_params=par, lib=lib)["A"]
+        assert np.abs(part - A_b[:, :, r0:]).max() <= TOL
+
+
 ALL_PINS = [pin_gamma1_is_sdpa, pin_full_window_is_sdpa, pin_zero_keys_closed_form,
             pin_window1_no_sink, pin_constant_values, pin_mask_structure,
-            pin_sampled_rows_are_dense, pin_gqa_repeat, pin_lemma1, pin_rows_agree]
-# The brute-force restatement is listed separately: the mutant test shows the
-# other pins catch every planted mistake without it.
-BRUTE_PINS = [pin_brute_force]
+            pin_sampled_rows_are_dense, pin_gqa_repeat, pin_lemma1, pin_rows_agree,
+            pin_smooth_reductions, pin_smooth_closed_forms]
+# The brute-force restatements are listed separately: the mutant test shows the
+# other pins catch every planted mistake without them.
+BRUTE_PINS = [pin_brute_force, pin_smooth_brute]

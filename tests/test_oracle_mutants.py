@@ -4,7 +4,9 @@ The mutants (ORACLE_MUTANT=n in oracle/delta_oracle.c) plant plausible
 mistakes: an off-by-one sink bound, a window one key too wide, the wrong GQA
 head mapping, a dropped 1/sqrt(d), a flipped Delta sign, the dense row taken
 over the sparse set, Delta taken against the current row instead of the
-sample, and a transposed K operand.  All of this runs on the CPU.
+sample, a transposed K operand, and three smoothing slips (EMA weights
+swapped, the filter's velocity gain replaced by its position gain, the
+interpolation weight one row ahead).  All of this runs on the CPU.
 """
 import os
 import tempfile
@@ -23,6 +25,9 @@ MUTANTS = {
     6: "dense row over the sparse set",
     7: "Delta against row i instead of its sample",
     8: "K read transposed",
+    9: "EMA weights swapped",
+    10: "filter velocity corrected with alpha",
+    11: "linear interpolation weight one row ahead",
 }
 
 _tmp = tempfile.mkdtemp(prefix="oracle_mutants_")
