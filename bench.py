@@ -14,8 +14,9 @@ dense kernel, then the sink+window kernel with the fused Delta epilogue.
                  recorded by the library on the launching stream
   cpu_baseline   the fp64 oracle on the host cores over a bounded sample
   dense_baseline gamma = 1 through the same kernels (dense causal attention)
-  variants       the Eq. 5 "recompute" output and a dense tail block of --tail
-                 rows (appendix "Implementation Details"), timed the same way
+  variants       the Eq. 5 "recompute" output, a dense tail block of --tail rows
+                 (appendix "Implementation Details") and the three Delta
+                 smoothing forms (appendix "Interpolation"), timed the same way
 
 ``--impl reference`` times the oracle as the reference arm.  Multi-GPU: one
 process per GPU (torchrun), independent sequences per rank, no collective on
@@ -237,19 +238,24 @@ def config_of(w, n_gpus):
 
 
 def time_variants(args, w, q, k, v, out, stream, restore):
-    """Median CUDA-event time of delta_attn_prefill_ex in the paper's ablation
-    forms: recompute (Eq. 5), Delta with a dense tail, recompute with a dense
-    tail.  The inputs are larger than L2, as in the main loop."""
+    """Median CUDA-event time of the prefill in the paper's ablation forms:
+    recompute (Eq. 5), Delta with a dense tail, recompute with a dense tail,
+    and the smoothed corrections (linear, EMA beta 0.5, the filter with
+    (0.2, 0.05, 0.0035)).  The inputs are larger than L2, as in the main loop."""
     from paper_2505_11254_gb300 import binding
     res = {}
-    for name, mode, tail in (("recompute", "recompute", 0), ("delta_tail", "delta", args.tail),
-                             ("recompute_tail", "recompute", args.tail)):
+    for name, mode, tail, sm, par in (("recompute", "recompute", 0, "none", ()),
+                                      ("delta_tail", "delta", args.tail, "none", ()),
+                                      ("recompute_tail", "recompute", args.tail, "none", ()),
+                                      ("smooth_linear", "delta", 0, "linear", ()),
+                                      ("smooth_ema", "delta", 0, "ema", (0.5,)),
+                                      ("smooth_abg", "delta", 0, "abg", (0.2, 0.05, 0.0035))):
         ws = binding.alloc_workspace(binding.workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window,
-                                                            w.gamma, mode, tail), q.device)
+                                                            w.gamma, mode, tail, smooth=sm), q.device)
 
         def call():
             binding.delta_attn_prefill(q, k, v, w.n_sink, w.window, w.gamma, out=out, workspace=ws, mode=mode,
-                                       tail_dense=tail)
+                                       tail_dense=tail, smooth=sm, smooth_params=par)
         for _ in range(3):
             call()
         torch.cuda.synchronize()
@@ -264,7 +270,8 @@ def time_variants(args, w, q, k, v, out, stream, restore):
         if binding.check() != binding.DA_OK:
             raise RuntimeError("device status after the %s timing" % name)
         ms = statistics.median(times)
-        res[name] = {"mode": mode, "tail_dense": tail, "ms": ms, "tokens_per_s": w.B * w.N / (ms / 1e3),
+        res[name] = {"mode": mode, "tail_dense": tail, "smooth": sm, "smooth_params": list(par), "ms": ms,
+                     "tokens_per_s": w.B * w.N / (ms / 1e3),
                      "tail_dense_pairs_per_head": flops.tail_pairs_per_head(w.N, tail)}
         del ws
     restore()  # `out` back to the Delta result for the spot check

@@ -113,6 +113,42 @@ int delta_attn_prefill_ex(const void* Q, const void* K, const void* V, void* O, 
                           int d, int n_sink, int64_t window, int gamma, int mode, int64_t tail_dense,
                           void* workspace, size_t ws_bytes, void* stream);
 
+/* Delta smoothing forms of delta_attn_prefill_smoothed() (appendix
+ * "Interpolation"). */
+typedef enum {
+    DA_SMOOTH_NONE = 0,    /* Eq. 6 as is                                          */
+    DA_SMOOTH_LINEAR = 1,  /* row i = k*gamma + r gets (1 - r/gamma) Delta_k +
+                              (r/gamma) Delta_{k+1}; the last group keeps Delta_k    */
+    DA_SMOOTH_EMA = 2,     /* c1 = beta in [0, 1]: over the rows, e_0 = Delta_0,
+                              e_i = (1 - beta) e_{i-1} + beta Delta_{floor(i/gamma)}   */
+    DA_SMOOTH_ABG = 3      /* c1, c2, c3 = the alpha, beta, gamma of Alg. 2's filter,
+                              run over the Delta vectors; row i gets the filter's
+                              output for its sample floor(i/gamma)                  */
+} da_smooth;
+
+/* Workspace bytes delta_attn_prefill_smoothed() needs: fp32 D and Delta rows,
+ * two fp32 basis vectors per sample, min(gamma, N) x 2 coefficients, split-K
+ * partials and tickets, and the dense tail's.  Returns a da_status. */
+int delta_attn_workspace_size_smoothed(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window,
+                                       int gamma, int smooth, int64_t tail_dense, size_t* bytes);
+
+/* The Eq. 6 prefill with the Delta corrections smoothed before they are added
+ * (appendix "Interpolation", Alg. 2).  Every row, sampled rows included, is
+ * written as bf16(S_i + corrected Delta); with DA_SMOOTH_NONE this is
+ * delta_attn_prefill_ex() in DA_MODE_DELTA.  Kernels, in stream order: the
+ * strided dense kernel (fp32 D), the strided sparse kernel (fp32 Delta_k =
+ * D_k - S_{k gamma}), the smoothing pass (one thread per head and column,
+ * sequential over the samples: the EMA carry between groups and the filter
+ * state), the sink+window kernel whose epilogue adds the smoothed correction,
+ * and the dense tail pass when tail_dense > 0.  c1..c3 must be finite; an EMA
+ * beta outside [0, 1] or an unknown form returns DA_ERR_INVALID_ARG.  The
+ * filter's stability is the caller's choice of coefficients.  Layouts,
+ * workspace, tail and errors as delta_attn_prefill_ex(). */
+int delta_attn_prefill_smoothed(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv,
+                                int64_t N, int d, int n_sink, int64_t window, int gamma, int smooth, double c1,
+                                double c2, double c3, int64_t tail_dense, void* workspace, size_t ws_bytes,
+                                void* stream);
+
 /* f*(Q,K,V) of Alg. 1 alone: StreamingLLM sink + window attention of every
  * row, written as bf16 to O_sparse.  When S_sampled is not NULL the fp32
  * sparse rows at the sampled rows k*gamma are also written (the operand

@@ -24,6 +24,7 @@ DA_ERR_TIMEOUT = -6
 DA_MODE_DELTA = 0
 DA_MODE_RECOMPUTE = 1
 _MODES = {"delta": DA_MODE_DELTA, "recompute": DA_MODE_RECOMPUTE}
+_SMOOTH = {"none": 0, "linear": 1, "ema": 2, "abg": 3}
 
 _lib = None
 
@@ -37,6 +38,9 @@ _SIGNATURES = {
     "delta_attn_prefill": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _sz, _p], _i),
     "delta_attn_workspace_size_ex": ([_i, _i, _i, _i64, _i, _i, _i64, _i, _i, _i64, ctypes.POINTER(_sz)], _i),
     "delta_attn_prefill_ex": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _i, _i64, _p, _sz, _p], _i),
+    "delta_attn_workspace_size_smoothed": ([_i, _i, _i, _i64, _i, _i, _i64, _i, _i, _i64, ctypes.POINTER(_sz)], _i),
+    "delta_attn_prefill_smoothed": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _i, ctypes.c_double,
+                                     ctypes.c_double, ctypes.c_double, _i64, _p, _sz, _p], _i),
     "delta_attn_prefill_events": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _sz, _p,
                                    ctypes.POINTER(_p), _i], _i),
     "sparse_window_attn": ([_p, _p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p], _i),
@@ -108,9 +112,15 @@ def _qkv_shape(q, k, v):
     return B, Hq, k.shape[1], N, d
 
 
-def workspace_size(B, Hq, Hkv, N, d, n_sink, window, gamma, mode="delta", tail_dense=0) -> int:
+def workspace_size(B, Hq, Hkv, N, d, n_sink, window, gamma, mode="delta", tail_dense=0, smooth="none") -> int:
     out = _sz(0)
-    if mode == "delta" and tail_dense == 0:
+    if smooth != "none":
+        if mode != "delta":
+            raise ValueError("smoothing applies to the Eq. 6 output")
+        _check(load().delta_attn_workspace_size_smoothed(B, Hq, Hkv, N, d, n_sink, window, gamma, _SMOOTH[smooth],
+                                                         tail_dense, ctypes.byref(out)),
+               "delta_attn_workspace_size_smoothed")
+    elif mode == "delta" and tail_dense == 0:
         _check(load().delta_attn_workspace_size(B, Hq, Hkv, N, d, n_sink, window, gamma, ctypes.byref(out)),
                "delta_attn_workspace_size")
     else:
@@ -131,16 +141,26 @@ def alloc_workspace(nbytes, device):
 
 
 def delta_attn_prefill(q, k, v, n_sink, window, gamma, out=None, workspace=None, stream=None, mode="delta",
-                       tail_dense=0):
+                       tail_dense=0, smooth="none", smooth_params=()):
     """Delta Attention prefill (Alg. 1 / Eq. 6) -> bf16 [B,Hq,N,d].
 
     ``mode="recompute"`` gives the Eq. 5 form and ``tail_dense=t`` makes the
-    last t rows dense (both through delta_attn_prefill_ex)."""
+    last t rows dense (both through delta_attn_prefill_ex); ``smooth`` =
+    "linear", "ema" (params (beta,)) or "abg" (params (alpha, beta, gamma))
+    smooths the corrections (delta_attn_prefill_smoothed)."""
     B, Hq, Hkv, N, d = _qkv_shape(q, k, v)
     if out is None:
         out = torch.empty_like(q)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
-    if mode == "delta" and tail_dense == 0:
+    if smooth != "none":
+        if mode != "delta":
+            raise ValueError("smoothing applies to the Eq. 6 output")
+        c1, c2, c3 = (tuple(float(x) for x in smooth_params) + (0.0, 0.0, 0.0))[:3]
+        _check(load().delta_attn_prefill_smoothed(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink,
+                                                  window, gamma, _SMOOTH[smooth], c1, c2, c3, tail_dense,
+                                                  _dptr(workspace), ws_bytes, _stream(stream)),
+               "delta_attn_prefill_smoothed")
+    elif mode == "delta" and tail_dense == 0:
         _check(load().delta_attn_prefill(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink,
                                          window, gamma, _dptr(workspace), ws_bytes, _stream(stream)),
                "delta_attn_prefill")

@@ -86,6 +86,10 @@ struct Plan {
   long long tail = 0;
   Params pt;
   size_t off_tail_part = 0, off_tail_ticket = 0;
+  // Delta smoothing: basis vectors per sample and the per-offset coefficients.
+  bool smooth = false;
+  size_t off_basis = 0, off_coef = 0;
+  int n_coef = 0;
 };
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -123,7 +127,7 @@ void plan_split_k(Params& p, int sms) {
 size_t ctrl_bytes(const Params& p) { return 4 * sizeof(unsigned long long) + (size_t)p.n_multi * sizeof(int); }
 
 Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma, int sms,
-               int64_t tail = 0) {
+               int64_t tail = 0, bool smooth = false) {
   Plan pl;
   Params& p = pl.p;
   p = Params{};
@@ -147,25 +151,35 @@ Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t win
   pl.grid_sparse = (long long)B * Hq * p.qtiles;
   pl.grid_dense = p.n_units;
   pl.fused_intile = gamma >= 2 && (BM % gamma) == 0 && (size_t)(BM / gamma) * d * sizeof(float) <= kSampleBufBytes;
-  pl.grid_ssparse = (gamma >= 2 && !pl.fused_intile) ? (long long)B * p.groups_per_b * p.mtiles : 0;
+  // Smoothing needs every Delta before any row is corrected: Delta is built
+  // in its own pass, for gamma = 1 as well.
+  pl.smooth = smooth;
+  pl.grid_ssparse = ((gamma >= 2 && !pl.fused_intile) || smooth) ? (long long)B * p.groups_per_b * p.mtiles : 0;
 
   const size_t rows_bytes = (size_t)B * Hq * p.n_s * d * sizeof(float);
   const size_t part_bytes = (size_t)p.n_multi * BM * (d + 2) * sizeof(float);
   const size_t ticket_bytes = ctrl_bytes(p);
   size_t off = 0;
-  if (gamma >= 2) {
+  if (gamma >= 2 || smooth) {
     pl.off_d = off;
     off += align256(rows_bytes);
-    if (!pl.fused_intile) {
+    if (!pl.fused_intile || smooth) {
       pl.off_delta = off;
       off += align256(rows_bytes);
     }
+  }
+  if (smooth) {
+    pl.n_coef = (int)std::min<int64_t>(gamma, N);
+    pl.off_basis = off;
+    off += align256(rows_bytes * kSmoothJ);
+    pl.off_coef = off;
+    off += align256((size_t)pl.n_coef * kSmoothJ * sizeof(float));
   }
   pl.off_part = off;
   off += align256(part_bytes);
   pl.off_ticket = off;
   off += align256(ticket_bytes);
-  if (tail > 0 && gamma >= 2) {
+  if (tail > 0 && (gamma >= 2 || smooth)) {
     pl.tail = tail;
     Params& t = pl.pt;
     t = p;
@@ -244,6 +258,19 @@ class ScopedWorkspace {
   bool owned_ = false, failed_ = false;
 };
 
+struct SmoothArgs {
+  int kind = DA_SMOOTH_NONE;
+  double c1 = 0, c2 = 0, c3 = 0;
+};
+
+int check_smooth(const SmoothArgs& sm, int mode) {
+  if (sm.kind < DA_SMOOTH_NONE || sm.kind > DA_SMOOTH_ABG) return DA_ERR_INVALID_ARG;
+  if (sm.kind != DA_SMOOTH_NONE && mode != DA_MODE_DELTA) return DA_ERR_INVALID_ARG;
+  if (!std::isfinite(sm.c1) || !std::isfinite(sm.c2) || !std::isfinite(sm.c3)) return DA_ERR_INVALID_ARG;
+  if (sm.kind == DA_SMOOTH_EMA && !(sm.c1 >= 0.0 && sm.c1 <= 1.0)) return DA_ERR_INVALID_ARG;
+  return DA_OK;
+}
+
 int check_variant(int mode, int64_t tail, int64_t N) {
   if (mode != DA_MODE_DELTA && mode != DA_MODE_RECOMPUTE) return DA_ERR_INVALID_ARG;
   if (tail < 0 || tail > N) return DA_ERR_INVALID_ARG;
@@ -252,8 +279,9 @@ int check_variant(int mode, int64_t tail, int64_t N) {
 
 // Kernel launches of one prefill call, in order.
 int prefill_kernels(const Plan& pl, int gamma, int mode) {
-  if (gamma == 1) return 1;
   const int tail = pl.tail > 0 ? 1 : 0;
+  if (pl.smooth) return 4 + tail;
+  if (gamma == 1) return 1;
   if (mode == DA_MODE_RECOMPUTE) return 2 + tail;
   return (pl.fused_intile ? 2 : 3) + tail;
 }
@@ -298,6 +326,19 @@ int delta_attn_workspace_size_ex(int B, int Hq, int Hkv, int64_t N, int d, int n
   return DA_OK;
 }
 
+int delta_attn_workspace_size_smoothed(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window,
+                                       int gamma, int smooth, int64_t tail_dense, size_t* bytes) {
+  if (!bytes) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
+  if (rc) return rc;
+  if ((rc = check_variant(DA_MODE_DELTA, tail_dense, N))) return rc;
+  if (smooth < DA_SMOOTH_NONE || smooth > DA_SMOOTH_ABG) return DA_ERR_INVALID_ARG;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  *bytes = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms, tail_dense, smooth != DA_SMOOTH_NONE).total;
+  return DA_OK;
+}
+
 int strided_dense_workspace_size(int B, int Hq, int Hkv, int64_t N, int d, int gamma, size_t* bytes) {
   if (!bytes) return DA_ERR_INVALID_ARG;
   int rc = check_shape(B, Hq, Hkv, N, d, 0, 1, gamma);
@@ -330,17 +371,19 @@ int delta_attn_plan_info(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, i
 }
 
 static int prefill_impl(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
-                        int d, int n_sink, int64_t window, int gamma, int mode, int64_t tail, void* workspace,
-                        size_t ws_bytes, void* stream, void* const* events, int n_events) {
+                        int d, int n_sink, int64_t window, int gamma, int mode, int64_t tail, const SmoothArgs& sm,
+                        void* workspace, size_t ws_bytes, void* stream, void* const* events, int n_events) {
   if (!Q || !K || !V || !O) return DA_ERR_INVALID_ARG;
   int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
   if (rc) return rc;
   if ((rc = check_variant(mode, tail, N))) return rc;
+  if ((rc = check_smooth(sm, mode))) return rc;
   if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(workspace))
     return DA_ERR_MISALIGNED;
   int sms = 0;
   if ((rc = check_device(&sms))) return rc;
-  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms, tail);
+  const bool smooth = sm.kind != DA_SMOOTH_NONE;
+  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms, tail, smooth);
   const int n_kernels = prefill_kernels(pl, gamma, mode);
   if (n_events != 0 && (events == nullptr || n_events != n_kernels + 1)) return DA_ERR_INVALID_ARG;
   if (workspace != nullptr && ws_bytes < pl.total) return DA_ERR_WORKSPACE;
@@ -348,7 +391,7 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   Params p = pl.p;
   if ((rc = status_ptr(&p.err))) return rc;
   Maps m;
-  if (!make_maps(&m, Q, K, V, p, d, gamma >= 2, true)) return DA_ERR_INVALID_ARG;
+  if (!make_maps(&m, Q, K, V, p, d, gamma >= 2 || smooth, true)) return DA_ERR_INVALID_ARG;
   CUtensorMap q_tail;
   if (pl.tail > 0 && !make_sample_map(&q_tail, Q, pl.pt, d)) return DA_ERR_INVALID_ARG;
 
@@ -382,6 +425,33 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   };
   if (!mark()) return DA_ERR_CUDA;
   cudaError_t e;
+  if (smooth) {
+    // Appendix "Interpolation": D, then every Delta_k, then the smoothing
+    // pass, then the sink+window pass adding the smoothed correction to
+    // every row (sampled rows included).
+    float* dbuf = reinterpret_cast<float*>(base + pl.off_d);
+    float* delta = reinterpret_cast<float*>(base + pl.off_delta);
+    float* basis = reinterpret_cast<float*>(base + pl.off_basis);
+    float* coef = reinterpret_cast<float*>(base + pl.off_coef);
+    p.d_out = dbuf;
+    e = launch<MODE_STRIDED_DENSE, EPI_DENSE_F32>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
+    if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
+    p.d_out = nullptr;
+    p.d_in = dbuf;
+    p.delta_out = delta;
+    e = launch<MODE_STRIDED_SPARSE, EPI_DELTA_BUILD>(d, m.qs, m.k, m.v, p, pl.grid_ssparse, s);
+    if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
+    p.delta_out = nullptr;
+    e = launch_delta_smooth(delta, basis, coef, (long long)B * Hq, p.n_s, d, gamma, pl.n_coef, sm.kind, sm.c1, sm.c2,
+                            sm.c3, s);
+    if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
+    p.out_bf16 = O;
+    p.smooth_basis = basis;
+    p.smooth_coef = coef;
+    e = launch<MODE_SPARSE, EPI_FUSED_SMOOTH>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+    if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
+    return run_tail();
+  }
   if (gamma == 1) {
     // Every row is a sampled row: the output is dense causal attention.
     p.out_bf16 = O;
@@ -423,22 +493,35 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
 int delta_attn_prefill(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
                        int d, int n_sink, int64_t window, int gamma, void* workspace, size_t ws_bytes,
                        void* stream) {
-  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, DA_MODE_DELTA, 0, workspace, ws_bytes,
-                      stream, nullptr, 0);
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, DA_MODE_DELTA, 0, SmoothArgs{},
+                      workspace, ws_bytes, stream, nullptr, 0);
 }
 
 int delta_attn_prefill_ex(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
                           int d, int n_sink, int64_t window, int gamma, int mode, int64_t tail_dense,
                           void* workspace, size_t ws_bytes, void* stream) {
-  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, mode, tail_dense, workspace, ws_bytes,
-                      stream, nullptr, 0);
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, mode, tail_dense, SmoothArgs{},
+                      workspace, ws_bytes, stream, nullptr, 0);
+}
+
+int delta_attn_prefill_smoothed(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv,
+                                int64_t N, int d, int n_sink, int64_t window, int gamma, int smooth, double c1,
+                                double c2, double c3, int64_t tail_dense, void* workspace, size_t ws_bytes,
+                                void* stream) {
+  SmoothArgs sm;
+  sm.kind = smooth;
+  sm.c1 = c1;
+  sm.c2 = c2;
+  sm.c3 = c3;
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, DA_MODE_DELTA, tail_dense, sm, workspace,
+                      ws_bytes, stream, nullptr, 0);
 }
 
 int delta_attn_prefill_events(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv,
                               int64_t N, int d, int n_sink, int64_t window, int gamma, void* workspace,
                               size_t ws_bytes, void* stream, void* const* events, int n_events) {
-  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, DA_MODE_DELTA, 0, workspace, ws_bytes,
-                      stream, events,
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, DA_MODE_DELTA, 0, SmoothArgs{},
+                      workspace, ws_bytes, stream, events,
                       n_events);
 }
 

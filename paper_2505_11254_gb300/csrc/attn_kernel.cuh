@@ -603,7 +603,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const long long bh = (long long)w.b * p.Hq + head;
       const float inv_l = (l_row > 0.f) ? 1.f / l_row : 0.f;
 
-      if (EPI == EPI_BF16 || EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA || EPI == EPI_DELTA_BUILD) {
+      if (EPI == EPI_BF16 || EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA || EPI == EPI_DELTA_BUILD ||
+          EPI == EPI_FUSED_SMOOTH) {
 #pragma unroll
         for (int c = 0; c < D; ++c) o[c] *= inv_l;
         const bool sampled = row_ok && is_sampled_row(row, p.gamma);
@@ -625,6 +626,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (EPI == EPI_BF16) {
               store_bf16x32(orow + q * 32, v);
               if (p.s_sampled != nullptr && sampled) store_f32x32(p.s_sampled + (bh * p.n_s + sample) * D + q * 32, v);
+            } else if (EPI == EPI_FUSED_SMOOTH) {
+              // every row, sampled or not: S_i + the smoothed correction of offset r
+              const int r = (int)(row - sample * p.gamma);
+              const float c0 = __ldg(p.smooth_coef + r * kSmoothJ), c1 = __ldg(p.smooth_coef + r * kSmoothJ + 1);
+              const float* bk = p.smooth_basis + (bh * p.n_s + sample) * (kSmoothJ * D) + q * 32;
+              float b0[32], b1[32];
+              load_f32x32(bk, b0);
+              load_f32x32(bk + D, b1);
+#pragma unroll
+              for (int c = 0; c < 32; ++c) b0[c] = fmaf(c1, b1[c], fmaf(c0, b0[c], v[c]));
+              store_bf16x32(orow + q * 32, b0);
             } else if (EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA) {
               float dk[32];
               load_f32x32(p.d_in + (bh * p.n_s + sample) * D + q * 32, dk);

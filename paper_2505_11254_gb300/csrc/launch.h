@@ -20,6 +20,8 @@ unsigned attn_smem_bytes(int d);
 
 cudaError_t launch_delta_apply(const void* o_sparse, const float* s_sampled, const float* d_sampled, void* o, int B,
                                int Hq, long long N, int d, int gamma, cudaStream_t s);
+cudaError_t launch_delta_smooth(const float* delta, float* basis, float* coef, long long BH, long long n_s, int d,
+                                int gamma, int n_coef, int kind, double c1, double c2, double c3, cudaStream_t s);
 cudaError_t launch_debug_mask(long long N, int n_sink, long long window, long long i0, long long i1,
                               unsigned char* out, cudaStream_t s);
 cudaError_t launch_debug_rowmap(long long N, int gamma, long long* sample_row, unsigned char* sampled,

@@ -31,7 +31,18 @@ enum Epi : int {
   EPI_DENSE_F32 = 3,     // sampled rows -> fp32 dense rows D_k
   EPI_DENSE_BF16 = 4,    // sampled rows (gamma = 1: every row) -> bf16 dense rows
   EPI_DELTA_BUILD = 5,   // sampled rows -> fp32 Delta_k = D_k - S_{k gamma}
+  EPI_FUSED_SMOOTH = 6,  // sparse rows -> bf16(S_i + sum_j coef[r][j] basis_k[j]), smoothed Delta
 };
+
+// Delta smoothing (appendix "Interpolation", Alg. 2): the correction of row
+// i = k gamma + r is coef[r][0] basis_k[0] + coef[r][1] basis_k[1].
+enum Smooth : int {
+  SMOOTH_NONE = 0,
+  SMOOTH_LINEAR = 1,  // basis (Delta_k, Delta_{k+1}), coef (1 - r/gamma, r/gamma)
+  SMOOTH_EMA = 2,     // basis (e_{k gamma - 1}, Delta_k), coef ((1-beta)^(r+1), 1 - (1-beta)^(r+1))
+  SMOOTH_ABG = 3,     // basis (filter output o_k), coef (1)
+};
+constexpr int kSmoothJ = 2;  // basis vectors per sample (the filter uses the first)
 
 struct Params {
   int B, Hq, Hkv, G;
@@ -59,6 +70,8 @@ struct Params {
   float* d_out;            // [B,Hq,n_s,d] fp32
   const float* delta_in;   // [B,Hq,n_s,d] fp32
   float* delta_out;        // [B,Hq,n_s,d] fp32
+  const float* smooth_basis;  // [B,Hq,n_s,kSmoothJ,d] fp32 (EPI_FUSED_SMOOTH)
+  const float* smooth_coef;   // [gamma][kSmoothJ] fp32 (EPI_FUSED_SMOOTH)
   float* partials;         // n_multi slots of BM*(d+2) fp32
   int* tickets;            // n_multi
   unsigned long long* counter;  // dynamic item counter (zeroed before the launch)
