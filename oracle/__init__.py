@@ -9,8 +9,8 @@ Two independent statements of the method live here:
   (causal softmax attention), the StreamingLLM sink + window set, Eq. 4
   (sampled rows k*gamma), Alg. 1 / Eq. 6 (Delta correction), Eq. 5
   ("recompute"), the appendix dense tail block and the appendix Delta
-  smoothing (linear interpolation, EMA, Alg. 2's alpha-beta-gamma filter),
-  all in double precision.
+  smoothing (linear interpolation, EMA, Alg. 2's alpha-beta-gamma filter)
+  and Eq. 2 decoding over the cache, all in double precision.
 * ``brute.py``: whole-matrix numpy evaluation (explicit N x N score matrix,
   -inf masks, matrix softmax, ``np.repeat`` of Delta) for small N.
 
@@ -53,6 +53,9 @@ def _load(path=None):
                                                    ci, ci, ci, ci, i64, i64, ci, ctypes.c_double, ctypes.c_double,
                                                    ctypes.c_double, i64, dp, dp, ci]
         lib.oracle_delta_attn_smoothed.restype = ci
+        lib.oracle_decode.argtypes = [u16p, u16p, u16p, ci, ci, ci, i64, ci, ctypes.POINTER(ctypes.c_int64), dp, dp,
+                                      ci]
+        lib.oracle_decode.restype = ci
         _libs[path] = lib
     return _libs[path]
 
@@ -152,6 +155,27 @@ def delta_attn(Q, K, V, n_sink, window, gamma, *, batches=None, heads=None, rows
     if rc != 0:
         raise ValueError("oracle_delta_attn_box failed (invalid arguments)")
     return {"A": A, "S": S, "D": D, "max_dev": dev.value}
+
+
+def decode(q, K, V, n_keys, nthreads=0, lib=None):
+    """Eq. 2 decoding: ``q`` [B,Hq,d] bf16 bits (one new token per sequence),
+    ``K``/``V`` caches [B,Hkv,L,d] bf16 bits holding the new token's key and
+    value at index n_keys[b]-1; ``n_keys`` [B] int.  Returns (out [B,Hq,d]
+    float64, max |sum p - 1|)."""
+    q, K, V = _u16(q), _u16(K), _u16(V)
+    if q.ndim != 3 or K.ndim != 4 or V.shape != K.shape or q.shape[0] != K.shape[0] or q.shape[2] != K.shape[3]:
+        raise ValueError("q [B,Hq,d], K,V [B,Hkv,L,d]")
+    B, Hq, d = q.shape
+    Hkv, L = K.shape[1], K.shape[2]
+    nk = np.ascontiguousarray(np.asarray(n_keys, dtype=np.int64).reshape(B))
+    out = np.empty((B, Hq, d), np.float64)
+    dev = ctypes.c_double(0.0)
+    rc = _load(lib).oracle_decode(_ptr(q, ctypes.c_uint16), _ptr(K, ctypes.c_uint16), _ptr(V, ctypes.c_uint16),
+                                  B, Hq, Hkv, L, d, _ptr(nk, ctypes.c_int64), _ptr(out, ctypes.c_double),
+                                  ctypes.byref(dev), nthreads)
+    if rc != 0:
+        raise ValueError("oracle_decode failed (invalid arguments)")
+    return out, dev.value
 
 
 def rows(Q, K, V, n_sink, window, gamma, bhi, nthreads=0, lib=None):

@@ -29,6 +29,8 @@
  *   - Appendix "Interpolation" and Alg. 2: smoothing of the Delta corrections
  *     (linear interpolation, EMA, alpha-beta-gamma filter) before they are
  *     added to the sparse rows.
+ *   - Eq. 2: decoding after the prefill, one new query per sequence attending
+ *     densely over the cached keys with its own key appended.
  *
  * Readings of the paper used here (each also listed in the design notes):
  *   - Rows are 0-based and the sample for row i is row floor(i/gamma)*gamma,
@@ -673,5 +675,72 @@ int oracle_delta_attn_smoothed(const uint16_t *Q, const uint16_t *K, const uint1
     free(delta);
     free(S);
     free(corr);
+    return rc;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Decoding (Eq. 2): the query of a newly generated token attends densely    */
+/* over the cache [K u k_new], [V u v_new].  The cache holds the new token's */
+/* key and value at index n_keys[b] - 1, so the keys are 0 .. n_keys[b] - 1. */
+
+typedef struct {
+    const uint16_t *q, *K, *V;
+    int B, Hq, Hkv, d;
+    int64_t L;
+    const int64_t *n_keys;
+    double *out;
+} decode_ctx;
+
+static void decode_item(void *vc, int64_t it, double *prob, double *dev)
+{
+    decode_ctx *c = (decode_ctx *)vc;
+    const int d = c->d;
+    const int b = (int)(it / c->Hq), h = (int)(it % c->Hq);
+    const int g = h / (c->Hq / c->Hkv);
+    const uint16_t *q = c->q + it * d;
+    const uint16_t *Kh = c->K + ((int64_t)b * c->Hkv + g) * c->L * d;
+    const uint16_t *Vh = c->V + ((int64_t)b * c->Hkv + g) * c->L * d;
+    const int64_t n = c->n_keys[b] - MUTANT(12);
+    const double tau = 1.0 / sqrt((double)d);
+    double *out = c->out + it * d;
+    double m = -INFINITY;
+    for (int64_t j = 0; j < n; ++j) {
+        double s = 0.0;
+        for (int x = 0; x < d; ++x) s += bf16_to_double(q[x]) * bf16_to_double(Kh[j * d + x]);
+        prob[j] = s * tau;
+        if (prob[j] > m) m = prob[j];
+    }
+    double Z = 0.0;
+    for (int64_t j = 0; j < n; ++j) {
+        prob[j] = exp(prob[j] - m);
+        Z += prob[j];
+    }
+    for (int x = 0; x < d; ++x) out[x] = 0.0;
+    double total = 0.0;
+    for (int64_t j = 0; j < n; ++j) {
+        const double pj = prob[j] / Z;
+        total += pj;
+        for (int x = 0; x < d; ++x) out[x] += pj * bf16_to_double(Vh[j * d + x]);
+    }
+    const double e = n > 0 ? fabs(total - 1.0) : 0.0;
+    if (e > *dev) *dev = e;
+}
+
+/*
+ * oracle_decode — q [B,Hq,d] (one new token per sequence), K and V caches
+ * [B,Hkv,L,d], n_keys[b] in [1, L] valid keys of sequence b; writes
+ * out [B,Hq,d].  Returns 0, or -1 on invalid arguments.
+ */
+int oracle_decode(const uint16_t *q, const uint16_t *K, const uint16_t *V, int B, int Hq, int Hkv, int64_t L,
+                  int d, const int64_t *n_keys, double *out, double *max_dev, int nthreads)
+{
+    if (!q || !K || !V || !n_keys || !out || B < 1 || Hq < 1 || Hkv < 1 || d < 1 || L < 1) return -1;
+    if (Hq % Hkv != 0) return -1;
+    for (int b = 0; b < B; ++b)
+        if (n_keys[b] < 1 || n_keys[b] > L) return -1;
+    decode_ctx c = {q, K, V, B, Hq, Hkv, d, L, n_keys, out};
+    double dev = 0.0;
+    int rc = run_pool(decode_item, &c, (int64_t)B * Hq, L, d, nthreads, &dev);
+    if (max_dev) *max_dev = dev;
     return rc;
 }

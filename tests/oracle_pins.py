@@ -17,6 +17,8 @@ What pins what:
   * GQA head mapping         -> explicit repetition of the KV heads.
   * Lemma 1                  -> the appendix inequality on every sample.
   * whole-matrix restatement -> the numpy brute force (oracle/brute.py).
+  * Eq. 2 decoding           -> the dense causal row at the token's position
+                                and torch scaled_dot_product_attention.
   * Delta smoothing          -> reductions to Eq. 6 (EMA beta = 1, filter
     (appendix Interpolation,    (1, 0, 0), linear at gamma = 1), fixed points
      Alg. 2)                    of a constant Delta, the EMA step response,
@@ -339,10 +341,32 @@ def pin_smooth_brute(lib=None):
         assert np.abs(part - A_b[:, :, r0:]).max() <= TOL
 
 
+def pin_decode(lib=None):
+    """Eq. 2 decoding of the token at position i over keys 0..i equals the
+    dense causal row i (Eq. 1, gamma = 1) and torch's scaled_dot_product_attention
+    of that single query over the same keys; a cache longer than n_keys is
+    ignored past n_keys."""
+    B, Hq, Hkv, N, d = 2, 4, 2, 50, 16
+    Q, K, V = rand_bits(60, (B, Hq, N, d)), rand_bits(61, (B, Hkv, N, d)), rand_bits(62, (B, Hkv, N, d))
+    dense = oracle.delta_attn(Q, K, V, 0, 1, 1, lib=lib)["A"]
+    for pos in ((0, 0), (7, 49), (31, 12)):
+        q = np.ascontiguousarray(np.stack([Q[b, :, pos[b]] for b in range(B)]))
+        out, dev = oracle.decode(q, K, V, [pos[0] + 1, pos[1] + 1], lib=lib)
+        assert dev <= 1e-12
+        for b in range(B):
+            assert np.abs(out[b] - dense[b, :, pos[b]]).max() <= TOL, pos
+            n = pos[b] + 1
+            Qt = torch.from_numpy(f64(q[b]))[None, :, None, :]
+            Kt = torch.from_numpy(f64(K[b, :, :n])).repeat_interleave(Hq // Hkv, dim=0)[None]
+            Vt = torch.from_numpy(f64(V[b, :, :n])).repeat_interleave(Hq // Hkv, dim=0)[None]
+            ref = torch.nn.functional.scaled_dot_product_attention(Qt, Kt, Vt).numpy()[0, :, 0]
+            assert np.abs(out[b] - ref).max() <= TOL
+
+
 ALL_PINS = [pin_gamma1_is_sdpa, pin_full_window_is_sdpa, pin_zero_keys_closed_form,
             pin_window1_no_sink, pin_constant_values, pin_mask_structure,
             pin_sampled_rows_are_dense, pin_gqa_repeat, pin_lemma1, pin_rows_agree,
-            pin_smooth_reductions, pin_smooth_closed_forms]
+            pin_smooth_reductions, pin_smooth_closed_forms, pin_decode]
 # The brute-force restatements are listed separately: the mutant test shows the
 # other pins catch every planted mistake without them.
 BRUTE_PINS = [pin_brute_force, pin_smooth_brute]

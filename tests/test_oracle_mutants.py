@@ -6,7 +6,8 @@ head mapping, a dropped 1/sqrt(d), a flipped Delta sign, the dense row taken
 over the sparse set, Delta taken against the current row instead of the
 sample, a transposed K operand, and three smoothing slips (EMA weights
 swapped, the filter's velocity gain replaced by its position gain, the
-interpolation weight one row ahead).  All of this runs on the CPU.
+interpolation weight one row ahead), and a decode that leaves out the new
+token's own key.  All of this runs on the CPU.
 """
 import os
 import tempfile
@@ -28,6 +29,7 @@ MUTANTS = {
     9: "EMA weights swapped",
     10: "filter velocity corrected with alpha",
     11: "linear interpolation weight one row ahead",
+    12: "decode without the new token's own key",
 }
 
 _tmp = tempfile.mkdtemp(prefix="oracle_mutants_")
