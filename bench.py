@@ -274,8 +274,42 @@ def time_variants(args, w, q, k, v, out, stream, restore):
                      "tokens_per_s": w.B * w.N / (ms / 1e3),
                      "tail_dense_pairs_per_head": flops.tail_pairs_per_head(w.N, tail)}
         del ws
+    res["decode"] = time_decode(w, q, k, v, stream)
     restore()  # `out` back to the Delta result for the spot check
     return res
+
+
+def time_decode(w, q, k, v, stream):
+    """Eq. 2 decoding of one new token per sequence over the whole N-token
+    cache (the workload's K and V; the last row plays the new token's key and
+    value): median CUDA-event time of delta_attn_decode, and the K/V bytes it
+    must read (each cached byte once, > L2) against the measured HBM copy
+    bandwidth."""
+    from paper_2505_11254_gb300 import binding
+    peaks, _ = load_peaks()
+    qd = q[:, :, -1, :].contiguous()
+    ws = binding.alloc_workspace(binding.decode_workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d), q.device)
+    od = torch.empty_like(qd)
+    for _ in range(3):
+        binding.decode(qd, k, v, out=od, workspace=ws)
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(20):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        binding.decode(qd, k, v, out=od, workspace=ws)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    if binding.check() != binding.DA_OK:
+        raise RuntimeError("device status after the decode timing")
+    ms = statistics.median(times)
+    kv_bytes = 2 * w.B * w.Hkv * w.N * w.d * 2
+    gbs = kv_bytes / (ms / 1e3) / 1e9
+    hbm = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
+    return {"context": w.N, "ms": ms, "tokens_per_s": w.B / (ms / 1e3), "kv_bytes": kv_bytes,
+            "achieved_gbs": gbs, "hbm_peak_gbs": hbm, "frac_of_hbm": gbs / hbm,
+            "note": "one token per sequence, all heads, split-K + merge kernels, launches included"}
 
 
 def run_ours(args, w, rep):

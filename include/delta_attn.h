@@ -189,6 +189,28 @@ int strided_dense_attn_noalloc(const void* Q, const void* K, const void* V, floa
 int delta_apply(const void* O_sparse, const float* S_sampled, const float* D_sampled, void* O, int B, int Hq,
                 int64_t N, int d, int gamma, void* stream);
 
+/* Workspace bytes delta_attn_decode() needs: one fp32 partial (o, max, sum)
+ * per query head and key range.  Returns a da_status. */
+int delta_attn_decode_workspace_size(int B, int Hq, int Hkv, int64_t max_keys, int d, size_t* bytes);
+
+/* Eq. 2: decoding after the prefill.  The query of one newly generated token
+ * per sequence attends densely over that sequence's cache, whose last valid
+ * entry is the new token's own key and value:
+ *   O[b,h,:] = softmax_j(q[b,h,:] . K[b,g,j,:] / sqrt(d)) V[b,g,j,:],
+ *   j = 0 .. lens[b] - 1, g = floor(h / (Hq/Hkv)).
+ *   q, O: [B, Hq, d] bf16; K, V: [B, Hkv, L, d] bf16 caches of capacity L
+ *   (rows past a sequence's length are never read); device pointers, 16-byte
+ *   aligned.  lens: device int64 [B], each in [1, L] (values outside are
+ *   clamped to [0, L]; a sequence with 0 keys gets a zero row), or NULL for
+ *   max_keys keys everywhere; 1 <= max_keys <= L bounds every lens[b] and
+ *   sizes the split.  Hq / Hkv <= 16, d in {64, 128}.
+ * Bound by HBM bandwidth (each cached byte is read once per step): CUDA-core
+ * kernel, split-K over key ranges with a second kernel merging them in a
+ * fixed order.  workspace may be NULL (stream-ordered allocation on `stream`).
+ * Returns a da_status; asynchronous on `stream`. */
+int delta_attn_decode(const void* q, const void* K, const void* V, const int64_t* lens, void* O, int B, int Hq,
+                      int Hkv, int64_t L, int64_t max_keys, int d, void* workspace, size_t ws_bytes, void* stream);
+
 /* Synchronises `stream`, returns and clears the device status word
  * (DA_OK, DA_ERR_TIMEOUT), or DA_ERR_CUDA if the stream reports an error. */
 int delta_attn_check(void* stream);

@@ -48,6 +48,8 @@ _SIGNATURES = {
     "strided_dense_attn": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _p, _sz, _p], _i),
     "strided_dense_attn_noalloc": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _p], _i),
     "delta_apply": ([_p, _p, _p, _p, _i, _i, _i64, _i, _i, _p], _i),
+    "delta_attn_decode_workspace_size": ([_i, _i, _i, _i64, _i, ctypes.POINTER(_sz)], _i),
+    "delta_attn_decode": ([_p, _p, _p, _p, _p, _i, _i, _i, _i64, _i64, _i, _p, _sz, _p], _i),
     "delta_attn_check": ([_p], _i),
     "delta_attn_status_string": ([_i], ctypes.c_char_p),
     "delta_attn_plan_info": ([_i, _i, _i, _i64, _i, _i, _i64, _i, ctypes.POINTER(_i64)], _i),
@@ -183,6 +185,37 @@ def delta_attn_prefill_events(q, k, v, n_sink, window, gamma, events, out=None, 
     _check(load().delta_attn_prefill_events(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink,
                                             window, gamma, _dptr(workspace), ws_bytes, _stream(stream), arr,
                                             len(events)), "delta_attn_prefill_events")
+    return out
+
+
+def decode_workspace_size(B, Hq, Hkv, max_keys, d) -> int:
+    out = _sz(0)
+    _check(load().delta_attn_decode_workspace_size(B, Hq, Hkv, max_keys, d, ctypes.byref(out)),
+           "delta_attn_decode_workspace_size")
+    return out.value
+
+
+def decode(q, k_cache, v_cache, lens=None, max_keys=None, out=None, workspace=None, stream=None):
+    """Eq. 2 decoding: ``q`` [B,Hq,d] bf16 (one new token per sequence),
+    ``k_cache``/``v_cache`` [B,Hkv,L,d] bf16 holding the new token's key and
+    value at index lens[b]-1; ``lens`` int64 CUDA tensor [B] or None (all
+    ``max_keys``, default L).  Returns bf16 [B,Hq,d]."""
+    if q.dim() != 3 or k_cache.dim() != 4 or v_cache.shape != k_cache.shape:
+        raise ValueError("q [B,Hq,d], caches [B,Hkv,L,d]")
+    for t in (q, k_cache, v_cache):
+        if not t.is_cuda or t.dtype != torch.bfloat16 or not t.is_contiguous():
+            raise ValueError("q and the caches must be contiguous bf16 CUDA tensors")
+    B, Hq, d = q.shape
+    Hkv, L = k_cache.shape[1], k_cache.shape[2]
+    if max_keys is None:
+        max_keys = L
+    if lens is not None and (lens.dtype != torch.int64 or not lens.is_cuda or lens.numel() != B):
+        raise ValueError("lens: int64 CUDA tensor [B]")
+    if out is None:
+        out = torch.empty_like(q)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(load().delta_attn_decode(_dptr(q), _dptr(k_cache), _dptr(v_cache), _dptr(lens), _dptr(out), B, Hq, Hkv,
+                                    L, max_keys, d, _dptr(workspace), ws_bytes, _stream(stream)), "delta_attn_decode")
     return out
 
 

@@ -271,6 +271,37 @@ int check_smooth(const SmoothArgs& sm, int mode) {
   return DA_OK;
 }
 
+// Split of the decode's key range: one wave of resident CTAs (the occupancy
+// of the kernel instance) over all (batch, KV head) pairs, each range a whole
+// number of ring chunks.
+struct DecodePlan {
+  int n_split = 1;
+  long long split_keys = 0;
+  size_t bytes = 0;
+};
+
+int check_decode(int B, int Hq, int Hkv, int64_t L, int64_t max_keys, int d) {
+  if (B < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || max_keys < 1 || L < max_keys) return DA_ERR_INVALID_ARG;
+  if ((int64_t)B * Hq > (int64_t(1) << 30) || L > (int64_t(1) << 40)) return DA_ERR_INVALID_ARG;
+  if (d != 64 && d != 128) return DA_ERR_UNSUPPORTED;
+  if (Hq / Hkv > 16) return DA_ERR_UNSUPPORTED;
+  return DA_OK;
+}
+
+DecodePlan make_decode_plan(int B, int Hq, int Hkv, int64_t max_keys, int d, int sms) {
+  DecodePlan dp;
+  const long long chunk = decode_keys_per_split();
+  const long long chunks = cdiv(max_keys, chunk);
+  const long long pairs = (long long)B * Hkv;
+  // at most one wave: a second, partial wave would run alone at the end
+  long long n = ((long long)decode_ctas_per_sm(d, Hq / Hkv) * std::max(sms, 1)) / pairs;
+  n = std::max<long long>(1, std::min(n, chunks));
+  dp.split_keys = cdiv(chunks, n) * chunk;
+  dp.n_split = (int)cdiv(max_keys, dp.split_keys);
+  dp.bytes = align256((size_t)pairs * dp.n_split * (Hq / Hkv) * (d + 2) * sizeof(float));
+  return dp;
+}
+
 int check_variant(int mode, int64_t tail, int64_t N) {
   if (mode != DA_MODE_DELTA && mode != DA_MODE_RECOMPUTE) return DA_ERR_INVALID_ARG;
   if (tail < 0 || tail > N) return DA_ERR_INVALID_ARG;
@@ -585,6 +616,51 @@ int delta_apply(const void* O_sparse, const float* S_sampled, const float* D_sam
   cudaError_t e = launch_delta_apply(O_sparse, S_sampled, D_sampled, O, B, Hq, N, d, gamma,
                                      static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? DA_OK : DA_ERR_CUDA;
+}
+
+int delta_attn_decode_workspace_size(int B, int Hq, int Hkv, int64_t max_keys, int d, size_t* bytes) {
+  if (!bytes) return DA_ERR_INVALID_ARG;
+  int rc = check_decode(B, Hq, Hkv, max_keys, max_keys, d);
+  if (rc) return rc;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  *bytes = make_decode_plan(B, Hq, Hkv, max_keys, d, sms).bytes;
+  return DA_OK;
+}
+
+int delta_attn_decode(const void* q, const void* K, const void* V, const int64_t* lens, void* O, int B, int Hq,
+                      int Hkv, int64_t L, int64_t max_keys, int d, void* workspace, size_t ws_bytes, void* stream) {
+  if (!q || !K || !V || !O) return DA_ERR_INVALID_ARG;
+  int rc = check_decode(B, Hq, Hkv, L, max_keys, d);
+  if (rc) return rc;
+  if (!aligned16(q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(workspace))
+    return DA_ERR_MISALIGNED;
+  if ((reinterpret_cast<uintptr_t>(lens) & 7u) != 0) return DA_ERR_MISALIGNED;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  const DecodePlan dp = make_decode_plan(B, Hq, Hkv, max_keys, d, sms);
+  if (workspace != nullptr && ws_bytes < dp.bytes) return DA_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  DecodeParams p{};
+  if ((rc = status_ptr(&p.err))) return rc;
+  ScopedWorkspace ws(workspace, dp.bytes, s);
+  if (ws.failed()) return DA_ERR_CUDA;
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.K = static_cast<const __nv_bfloat16*>(K);
+  p.V = static_cast<const __nv_bfloat16*>(V);
+  p.lens = reinterpret_cast<const long long*>(lens);
+  p.max_keys = max_keys;
+  p.L = L;
+  p.B = B;
+  p.Hq = Hq;
+  p.Hkv = Hkv;
+  p.G = Hq / Hkv;
+  p.D = d;
+  p.n_split = dp.n_split;
+  p.split_keys = dp.split_keys;
+  p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
+  p.part = reinterpret_cast<float*>(ws.get());
+  return launch_decode(p, O, s) == cudaSuccess ? DA_OK : DA_ERR_CUDA;
 }
 
 int delta_attn_check(void* stream) {

@@ -1,0 +1,362 @@
+// decode.cu — Eq. 2: decoding after the sparse prefill.  The query of each
+// newly generated token attends densely over the whole cache [K u k_new],
+// [V u v_new] of its sequence (the new key and value already appended).
+//
+// The step reads every cached key and value once and does 4*d FLOPs per key
+// and query head, so it is bound by HBM bandwidth, not by the tensor cores
+// (with one query row per head there is no tile to fill).  Design:
+//   * split-K: a CTA per (batch, KV head, key range) handles the G query
+//     heads of the KV group together, so each K/V byte is read once;
+//   * a producer warp streams 16-key K and V chunks (contiguous rows) with
+//     cp.async.bulk into a 4-stage shared-memory ring completed on mbarriers
+//     (32 KB at d = 128, so several CTAs share an SM and each SM sub-partition
+//     interleaves their consumer warps while the next chunks load); the key
+//     range is split so that one wave of CTAs fills every SM;
+//   * four consumer warps take whole chunks in turn.  A lane owns d/32 channels
+//     of every head; for 32/GP keys x GP heads (GP = G rounded up to a power
+//     of two) it forms 32 partial dot products, and a butterfly of 31 shuffles
+//     leaves lane l with the full score of pair l (key l / GP, head l % GP);
+//     the online softmax (running max and sum per head, exp2 with log2(e)/sqrt(d)
+//     folded into q) then broadcasts each weight to the lanes for P.V;
+//   * the warps' partial states are merged in shared memory and written as
+//     (unnormalised o, max, sum) per split; a second kernel merges the splits
+//     in a fixed order (deterministic) and writes bf16.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "launch.h"
+#include "ptx.cuh"
+#include "wait.cuh"
+
+namespace da {
+namespace {
+
+constexpr int kDecWarps = 4;                        // consumer warps
+constexpr int kDecThreads = (kDecWarps + 1) * 32;   // + the producer warp
+constexpr int kDecChunk = 16;                       // keys per ring stage
+constexpr int kDecStages = 4;
+// Chunk i goes to stage i % kDecStages and to consumer warp i % kDecWarps.
+// With kDecStages a multiple of kDecWarps every phase of a stage is consumed
+// by the same warp in order, so a parity wait can never be satisfied by a
+// phase two behind the one it wants.
+static_assert(kDecStages % kDecWarps == 0, "each stage must belong to one consumer warp");
+
+template <int D>
+constexpr int dec_smem_bytes() {
+  return kDecStages * 2 * kDecChunk * D * 2 + 1024;
+}
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+
+template <int CPL>
+__device__ __forceinline__ void load_row(const __nv_bfloat16* row, int lane, float (&f)[CPL]) {
+  if constexpr (CPL == 4) {
+    const uint2 u = *reinterpret_cast<const uint2*>(row + lane * 4);
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+    f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y;
+  } else {
+    const uint32_t u = *reinterpret_cast<const uint32_t*>(row + lane * 2);
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u));
+    f[0] = a.x; f[1] = a.y;
+  }
+}
+
+template <int D, int GP>
+__global__ void __launch_bounds__(kDecThreads) decode_kernel(DecodeParams p) {
+  constexpr int CPL = D / 32;   // channels per lane
+  constexpr int KW = 32 / GP;   // keys per inner iteration
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __nv_bfloat16* ring = reinterpret_cast<__nv_bfloat16*>(smem);  // [stage][K|V][kDecChunk][D]
+  __shared__ uint64_t full[kDecStages], empty[kDecStages];
+  __shared__ volatile int abort_sh;
+  __shared__ float wm[kDecWarps][GP], wl[kDecWarps][GP];
+  __shared__ float wo[kDecWarps][GP][D];
+
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const long long unit = blockIdx.x;
+  const int s = (int)(unit % p.n_split);
+  const long long bg = unit / p.n_split;  // b * Hkv + g
+  const int b = (int)(bg / p.Hkv), g = (int)(bg % p.Hkv);
+  long long n = p.lens != nullptr ? p.lens[b] : p.max_keys;
+  n = n < 0 ? 0 : (n > p.L ? p.L : n);
+  const long long k_begin = (long long)s * p.split_keys;
+  const long long k_end = (k_begin + p.split_keys < n) ? k_begin + p.split_keys : n;
+  const int nc = k_end > k_begin ? (int)((k_end - k_begin + kDecChunk - 1) / kDecChunk) : 0;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kDecStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    abort_sh = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+
+  const __nv_bfloat16* Kg = p.K + (bg * p.L) * D;
+  const __nv_bfloat16* Vg = p.V + (bg * p.L) * D;
+  if (warp == kDecWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int issued = 0;
+      for (int i = 0; i < nc; ++i) {
+        const int st = i % kDecStages;
+        if (i >= kDecStages && !wait_bounded(&empty[st], ((i / kDecStages) - 1) & 1, &abort_sh, p.err)) break;
+        const long long k0 = k_begin + (long long)i * kDecChunk;
+        const long long nk = (k_end - k0 < kDecChunk) ? k_end - k0 : kDecChunk;
+        const uint32_t bytes = (uint32_t)(nk * D * 2);
+        mbar_arrive_expect_tx(&full[st], 2 * bytes);
+        bulk_g2s(ring + (size_t)(st * 2) * kDecChunk * D, Kg + k0 * D, bytes, &full[st]);
+        bulk_g2s(ring + (size_t)(st * 2 + 1) * kDecChunk * D, Vg + k0 * D, bytes, &full[st]);
+        ++issued;
+      }
+      // The ring must be quiet before the CTA exits: wait for the latest
+      // phase of every stage still in use.
+      for (int i = (issued > kDecStages ? issued - kDecStages : 0); i < issued; ++i)
+        wait_drain(&full[i % kDecStages], (i / kDecStages) & 1, p.err);
+    }
+    return;
+  }
+
+  // -------------------------------------------------------------- consumers
+  const int G = p.G;
+  float qv[GP][CPL];
+#pragma unroll
+  for (int h = 0; h < GP; ++h) {
+    if (h < G) {
+      load_row<CPL>(p.q + ((long long)b * p.Hq + (long long)g * G + h) * D, lane, qv[h]);
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) qv[h][c] *= p.scale_log2;
+    } else {
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) qv[h][c] = 0.f;
+    }
+  }
+  float o[GP][CPL];
+#pragma unroll
+  for (int h = 0; h < GP; ++h)
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) o[h][c] = 0.f;
+  float m_own = -INFINITY, l_own = 0.f;  // running max / sum of head lane % GP
+
+  for (int i = warp; i < nc; i += kDecWarps) {
+    const int st = i % kDecStages;
+    if (!__all_sync(0xffffffffu, wait_bounded(&full[st], (i / kDecStages) & 1, &abort_sh, p.err))) break;
+    const __nv_bfloat16* Ks = ring + (size_t)(st * 2) * kDecChunk * D;
+    const __nv_bfloat16* Vs = ring + (size_t)(st * 2 + 1) * kDecChunk * D;
+    const long long k0 = k_begin + (long long)i * kDecChunk;
+    const int nk = (int)((k_end - k0 < kDecChunk) ? k_end - k0 : kDecChunk);
+#pragma unroll 1
+    for (int kb = 0; kb < nk; kb += KW) {
+      float acc[32];
+#pragma unroll
+      for (int kk = 0; kk < KW; ++kk) {
+        float kf[CPL];
+        load_row<CPL>(Ks + (size_t)(kb + kk) * D, lane, kf);  // rows past nk hold stale data: masked below
+#pragma unroll
+        for (int h = 0; h < GP; ++h) {
+          float a = qv[h][0] * kf[0];
+#pragma unroll
+          for (int c = 1; c < CPL; ++c) a = fmaf(qv[h][c], kf[c], a);
+          acc[kk * GP + h] = a;
+        }
+      }
+      // butterfly: lane l ends with the sum over lanes of acc[l]
+#pragma unroll
+      for (int half = 16; half >= 1; half >>= 1) {
+        const bool upper = (lane & half) != 0;
+#pragma unroll
+        for (int e = 0; e < half; ++e) {
+          const float send = upper ? acc[e] : acc[e + half];
+          const float keep = upper ? acc[e + half] : acc[e];
+          acc[e] = keep + __shfl_xor_sync(0xffffffffu, send, half);
+        }
+      }
+      const bool key_ok = kb + lane / GP < nk;
+      const float sc = key_ok ? acc[0] : -INFINITY;
+      float mh = sc;
+#pragma unroll
+      for (int off = GP; off < 32; off <<= 1) mh = fmaxf(mh, __shfl_xor_sync(0xffffffffu, mh, off));
+      const float m_new = fmaxf(m_own, mh);
+      const float mu = (m_new == -INFINITY) ? 0.f : m_new;
+      const float pr = ex2(sc - mu);
+      const float alpha = ex2(m_own - mu);
+      float ps = pr;
+#pragma unroll
+      for (int off = GP; off < 32; off <<= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
+      l_own = l_own * alpha + ps;
+      // O is rescaled only when some head's running max grew (alpha = 1
+      // exactly otherwise), which after the first keys is rare.
+      if (__any_sync(0xffffffffu, m_new != m_own)) {
+#pragma unroll
+        for (int h = 0; h < GP; ++h) {
+          const float ah = __shfl_sync(0xffffffffu, alpha, h);
+#pragma unroll
+          for (int c = 0; c < CPL; ++c) o[h][c] *= ah;
+        }
+      }
+      m_own = m_new;
+#pragma unroll
+      for (int kk = 0; kk < KW; ++kk) {
+        if (kb + kk < nk) {  // warp-uniform
+          float vf[CPL];
+          load_row<CPL>(Vs + (size_t)(kb + kk) * D, lane, vf);
+#pragma unroll
+          for (int h = 0; h < GP; ++h) {
+            const float pk = __shfl_sync(0xffffffffu, pr, kk * GP + h);
+            const uint64_t pk2 = f2_pack(pk, pk);
+#pragma unroll
+            for (int c = 0; c < CPL; c += 2) {
+              float lo, hi;
+              f2_unpack(f2_fma(pk2, f2_pack(vf[c], vf[c + 1]), f2_pack(o[h][c], o[h][c + 1])), lo, hi);
+              o[h][c] = lo;
+              o[h][c + 1] = hi;
+            }
+          }
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[st]);
+  }
+
+  // merge the four warps' states, then write this split's partial
+  if (lane < GP) {
+    wm[warp][lane] = m_own;
+    wl[warp][lane] = l_own;
+  }
+#pragma unroll
+  for (int h = 0; h < GP; ++h)
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) wo[warp][h][lane * CPL + c] = o[h][c];
+  asm volatile("bar.sync 1, %0;" ::"n"(kDecWarps * 32) : "memory");
+  float* part = p.part + (size_t)unit * G * (D + 2);
+  for (int idx = threadIdx.x; idx < G * D; idx += kDecWarps * 32) {
+    const int h = idx / D, c = idx % D;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kDecWarps; ++w) M = fmaxf(M, wm[w][h]);
+    const float Mu = (M == -INFINITY) ? 0.f : M;
+    float acc = 0.f, lsum = 0.f;
+#pragma unroll
+    for (int w = 0; w < kDecWarps; ++w) {
+      const float f = ex2(wm[w][h] - Mu);
+      acc = fmaf(wo[w][h][c], f, acc);
+      lsum = fmaf(wl[w][h], f, lsum);
+    }
+    part[h * (D + 2) + c] = acc;
+    if (c == 0) {
+      part[h * (D + 2) + D] = M;
+      part[h * (D + 2) + D + 1] = lsum;
+    }
+  }
+}
+
+// One thread per (batch, query head, column): the splits in order.
+__global__ void __launch_bounds__(128) decode_merge_kernel(const float* __restrict__ part, __nv_bfloat16* out,
+                                                           long long rows, int Hq, int Hkv, int G, int n_split,
+                                                           int d) {
+  const long long t = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  if (t >= rows * d) return;
+  const long long bh = t / d;
+  const int c = (int)(t % d);
+  const long long b = bh / Hq;
+  const int h = (int)(bh % Hq), g = h / G, hh = h % G;
+  const float* base = part + ((size_t)(b * Hkv + g) * n_split) * G * (d + 2) + (size_t)hh * (d + 2);
+  const size_t stride = (size_t)G * (d + 2);
+  float M = -INFINITY;
+  for (int s = 0; s < n_split; ++s) M = fmaxf(M, base[s * stride + d]);
+  const float Mu = (M == -INFINITY) ? 0.f : M;
+  float acc = 0.f, lsum = 0.f;
+  for (int s = 0; s < n_split; ++s) {
+    const float f = ex2(base[s * stride + d] - Mu);
+    acc = fmaf(base[s * stride + c], f, acc);
+    lsum = fmaf(base[s * stride + d + 1], f, lsum);
+  }
+  out[t] = __float2bfloat16_rn(lsum > 0.f ? acc / lsum : 0.f);
+}
+
+template <int D, int GP>
+cudaError_t launch_decode_t(const DecodeParams& p, long long units, cudaStream_t s) {
+  auto k = decode_kernel<D, GP>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, dec_smem_bytes<D>());
+  if (e != cudaSuccess) return e;
+  k<<<(unsigned)units, kDecThreads, dec_smem_bytes<D>(), s>>>(p);
+  return cudaGetLastError();
+}
+
+template <int D>
+cudaError_t launch_decode_d(const DecodeParams& p, long long units, cudaStream_t s) {
+  const int G = p.G;
+  if (G <= 1) return launch_decode_t<D, 1>(p, units, s);
+  if (G <= 2) return launch_decode_t<D, 2>(p, units, s);
+  if (G <= 4) return launch_decode_t<D, 4>(p, units, s);
+  if (G <= 8) return launch_decode_t<D, 8>(p, units, s);
+  return launch_decode_t<D, 16>(p, units, s);
+}
+
+}  // namespace
+
+int decode_keys_per_split() { return kDecChunk; }
+
+// Queried once per kernel instance (the answer is the same on every GB300;
+// concurrent first calls compute the same value).
+template <int D, int GP>
+int ctas_per_sm_t() {
+  static int cached = 0;
+  if (cached > 0) return cached;
+  int n = 0;
+  auto k = decode_kernel<D, GP>;
+  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, dec_smem_bytes<D>()) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, kDecThreads, dec_smem_bytes<D>()) != cudaSuccess)
+    return 1;
+  cached = n > 0 ? n : 1;
+  return cached;
+}
+
+template <int D>
+int ctas_per_sm_d(int G) {
+  if (G <= 1) return ctas_per_sm_t<D, 1>();
+  if (G <= 2) return ctas_per_sm_t<D, 2>();
+  if (G <= 4) return ctas_per_sm_t<D, 4>();
+  if (G <= 8) return ctas_per_sm_t<D, 8>();
+  return ctas_per_sm_t<D, 16>();
+}
+
+int decode_ctas_per_sm(int d, int G) { return d == 64 ? ctas_per_sm_d<64>(G) : ctas_per_sm_d<128>(G); }
+
+cudaError_t launch_decode(const DecodeParams& p, void* out, cudaStream_t s) {
+  const long long units = (long long)p.B * p.Hkv * p.n_split;
+  if (units <= 0 || units > 0x7fffffffLL) return cudaErrorInvalidValue;
+  cudaError_t e = p.D == 64 ? launch_decode_d<64>(p, units, s) : launch_decode_d<128>(p, units, s);
+  if (e != cudaSuccess) return e;
+  const long long rows = (long long)p.B * p.Hq;
+  const long long threads = rows * p.D;
+  decode_merge_kernel<<<(unsigned)((threads + 127) / 128), 128, 0, s>>>(
+      p.part, static_cast<__nv_bfloat16*>(out), rows, p.Hq, p.Hkv, p.G, p.n_split, p.D);
+  return cudaGetLastError();
+}
+
+}  // namespace da

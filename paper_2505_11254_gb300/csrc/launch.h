@@ -2,6 +2,7 @@
 // attn_*.cu so the kernels compile in parallel translation units).
 #pragma once
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "tiles.cuh"
@@ -22,6 +23,24 @@ cudaError_t launch_delta_apply(const void* o_sparse, const float* s_sampled, con
                                int Hq, long long N, int d, int gamma, cudaStream_t s);
 cudaError_t launch_delta_smooth(const float* delta, float* basis, float* coef, long long BH, long long n_s, int d,
                                 int gamma, int n_coef, int kind, double c1, double c2, double c3, cudaStream_t s);
+// Eq. 2 decoding over the cache (decode.cu).
+struct DecodeParams {
+  const __nv_bfloat16* q;  // [B, Hq, D]
+  const __nv_bfloat16* K;  // [B, Hkv, L, D]
+  const __nv_bfloat16* V;  // [B, Hkv, L, D]
+  const long long* lens;   // [B] valid keys per sequence (device), or null: max_keys each
+  long long max_keys, L;
+  int B, Hq, Hkv, G, D;
+  int n_split;             // key ranges per (batch, KV head)
+  long long split_keys;    // keys per range, a multiple of decode_keys_per_split()
+  float scale_log2;        // log2(e) / sqrt(D)
+  float* part;             // [B * Hkv * n_split][G][D + 2]: unnormalised o, max, sum
+  int* err;                // device status word
+};
+int decode_keys_per_split();
+int decode_ctas_per_sm(int d, int G);  // resident decode CTAs per SM (occupancy)
+cudaError_t launch_decode(const DecodeParams& p, void* out, cudaStream_t s);
+
 cudaError_t launch_debug_mask(long long N, int n_sink, long long window, long long i0, long long i1,
                               unsigned char* out, cudaStream_t s);
 cudaError_t launch_debug_rowmap(long long N, int gamma, long long* sample_row, unsigned char* sampled,

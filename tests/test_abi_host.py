@@ -94,3 +94,27 @@ def test_prefill_ex_rejects_bad_mode_and_tail(mode, tail):
     sz = ctypes.c_size_t(0)
     assert lib.delta_attn_workspace_size_ex(1, 4, 2, 256, 128, 4, 64, 16, mode, tail, ctypes.byref(sz)) == \
         binding.DA_ERR_INVALID_ARG
+
+
+def test_decode_rejects_bad_arguments():
+    """Eq. 2 decode: NULL or misaligned pointers, L < max_keys, max_keys < 1,
+    Hq % Hkv != 0, G > 16 and an unsupported head dimension are rejected
+    before any device call."""
+    lib = binding.load()
+    ok = dict(q=_FAKE, K=_FAKE, V=_FAKE, lens=None, O=_FAKE, B=1, Hq=8, Hkv=2, L=100, mk=100, d=128)
+
+    def call(**kw):
+        a = dict(ok)
+        a.update(kw)
+        return lib.delta_attn_decode(a["q"], a["K"], a["V"], a["lens"], a["O"], a["B"], a["Hq"], a["Hkv"], a["L"],
+                                     a["mk"], a["d"], None, 0, None)
+    assert call(q=None) == binding.DA_ERR_INVALID_ARG
+    assert call(L=50) == binding.DA_ERR_INVALID_ARG
+    assert call(mk=0) == binding.DA_ERR_INVALID_ARG
+    assert call(Hq=7) == binding.DA_ERR_INVALID_ARG
+    assert call(Hq=34, Hkv=2) == binding.DA_ERR_UNSUPPORTED
+    assert call(d=96) == binding.DA_ERR_UNSUPPORTED
+    assert call(K=_FAKE + 8) == binding.DA_ERR_MISALIGNED
+    assert call(lens=_FAKE + 4) == binding.DA_ERR_MISALIGNED
+    sz = ctypes.c_size_t(0)
+    assert lib.delta_attn_decode_workspace_size(1, 8, 2, 0, 128, ctypes.byref(sz)) == binding.DA_ERR_INVALID_ARG
