@@ -7,18 +7,18 @@
 // (with one query row per head there is no tile to fill).  Design:
 //   * split-K: a CTA per (batch, KV head, key range) handles the G query
 //     heads of the KV group together, so each K/V byte is read once;
-//   * a producer warp streams 16-key K and V chunks (contiguous rows) with
-//     cp.async.bulk into a 4-stage shared-memory ring completed on mbarriers
-//     (32 KB at d = 128, so several CTAs share an SM and each SM sub-partition
-//     interleaves their consumer warps while the next chunks load); the key
-//     range is split so that one wave of CTAs fills every SM;
-//   * four consumer warps take whole chunks in turn.  A lane owns d/32 channels
-//     of every head; for 32/GP keys x GP heads (GP = G rounded up to a power
-//     of two) it forms 32 partial dot products, and a butterfly of 31 shuffles
-//     leaves lane l with the full score of pair l (key l / GP, head l % GP);
-//     the online softmax (running max and sum per head, exp2 with log2(e)/sqrt(d)
-//     folded into q) then broadcasts each weight to the lanes for P.V;
-//   * the warps' partial states are merged in shared memory and written as
+//   * a producer warp streams 32-key K and V chunks (contiguous rows) with
+//     cp.async.bulk into a 4-stage shared-memory ring completed on mbarriers;
+//     the key range is split so that one wave of CTAs fills every SM;
+//   * four consumer warps take whole chunks in turn.  Inside a warp, groups
+//     of LPK lanes work on different keys (layout in DecLayout): a lane holds
+//     a slice of the channels of q and o for every head (GP = G rounded up to
+//     a power of two), forms partial dot products for its group's keys, and
+//     a reduce-scatter over the group's lanes completes the scores; the online
+//     softmax (running max and sum per head and group, exp2 with
+//     log2(e)/sqrt(d) folded into q) then broadcasts each weight to the
+//     group's lanes for P.V with packed fp32 FMAs;
+//   * the (warp, group) partial states are merged in shared memory and written as
 //     (unnormalised o, max, sum) per split; a second kernel merges the splits
 //     in a fixed order (deterministic) and writes bf16.
 #include <cuda_bf16.h>
@@ -34,8 +34,10 @@ namespace {
 
 constexpr int kDecWarps = 4;                        // consumer warps
 constexpr int kDecThreads = (kDecWarps + 1) * 32;   // + the producer warp
-constexpr int kDecChunk = 16;                       // keys per ring stage
+constexpr int kDecChunk = 32;                       // keys per ring stage
 constexpr int kDecStages = 4;
+constexpr int kDecQORegs = 64;  // registers per lane for its slices of q and o
+constexpr int kDecMinCtas = 2;  // CTAs per SM the register allocation must allow
 // Chunk i goes to stage i % kDecStages and to consumer warp i % kDecWarps.
 // With kDecStages a multiple of kDecWarps every phase of a stage is consumed
 // by the same warp in order, so a parity wait can never be satisfied by a
@@ -68,31 +70,76 @@ __device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
   return d;
 }
 
-template <int CPL>
-__device__ __forceinline__ void load_row(const __nv_bfloat16* row, int lane, float (&f)[CPL]) {
-  if constexpr (CPL == 4) {
-    const uint2 u = *reinterpret_cast<const uint2*>(row + lane * 4);
-    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
-    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
-    f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y;
-  } else {
-    const uint32_t u = *reinterpret_cast<const uint32_t*>(row + lane * 2);
-    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u));
-    f[0] = a.x; f[1] = a.y;
+// Lane layout of a consumer warp for GP (padded) query heads of width D:
+//   LPK lanes share one key (a group; NG = 32 / LPK groups per warp run on
+//   different keys), each lane holding CPL = D / LPK channels of q and o for
+//   all GP heads (2 * GP * CPL <= kDecQORegs registers, so that two CTAs fit
+//   an SM's register file);
+//   a group forms the partial dot products of KG keys x GP heads over its
+//   channels (N = KG * GP values per lane) and reduce-scatters them over its
+//   LPK lanes, leaving R = N / LPK complete scores per lane;
+//   channels are dealt in 16-byte pieces, piece p of a row to lane p % LPK,
+//   so the lanes of a quarter warp read one contiguous 128-byte span.
+template <int D, int GP>
+struct DecLayout {
+  static constexpr int cl(int x, int lo, int hi) { return x < lo ? lo : (x > hi ? hi : x); }
+  static constexpr int mn(int a, int b) { return a < b ? a : b; }
+  static constexpr int LPK = cl(2 * GP * D / kDecQORegs, 2, 32);
+  static constexpr int NG = 32 / LPK;
+  static constexpr int CPL = D / LPK;
+  static constexpr int R = mn(mn(4, GP), 32 / LPK);
+  static constexpr int N = LPK * R;
+  static constexpr int KG = N / GP;
+  static constexpr int KEYS = NG * KG;           // keys per warp iteration
+  static constexpr int PS = CPL < 8 ? CPL : 8;   // channels per piece
+  static constexpr int T = CPL / PS;             // pieces per lane
+  static_assert(KG >= 1 && N % GP == 0 && N % LPK == 0, "layout");
+  static_assert(kDecChunk % KEYS == 0, "a chunk holds whole iterations");
+};
+
+// Channels of one row slice (T pieces of PS channels) as floats.
+template <int D, int GP>
+__device__ __forceinline__ void load_slice(const __nv_bfloat16* row, int sub, float* f) {
+  using L = DecLayout<D, GP>;
+#pragma unroll
+  for (int t = 0; t < L::T; ++t) {
+    const __nv_bfloat16* src = row + (sub + L::LPK * t) * L::PS;
+    if constexpr (L::PS == 8) {
+      const uint4 u = *reinterpret_cast<const uint4*>(src);
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        f[t * 8 + 2 * e] = __uint_as_float(w[e] << 16);
+        f[t * 8 + 2 * e + 1] = __uint_as_float(w[e] & 0xffff0000u);
+      }
+    } else if constexpr (L::PS == 4) {
+      const uint2 u = *reinterpret_cast<const uint2*>(src);
+      f[t * 4 + 0] = __uint_as_float(u.x << 16);
+      f[t * 4 + 1] = __uint_as_float(u.x & 0xffff0000u);
+      f[t * 4 + 2] = __uint_as_float(u.y << 16);
+      f[t * 4 + 3] = __uint_as_float(u.y & 0xffff0000u);
+    } else {
+      static_assert(L::PS == 2, "pieces of 2, 4 or 8 channels");
+      const uint32_t u = *reinterpret_cast<const uint32_t*>(src);
+      f[t * 2 + 0] = __uint_as_float(u << 16);
+      f[t * 2 + 1] = __uint_as_float(u & 0xffff0000u);
+    }
   }
 }
 
 template <int D, int GP>
-__global__ void __launch_bounds__(kDecThreads) decode_kernel(DecodeParams p) {
-  constexpr int CPL = D / 32;   // channels per lane
-  constexpr int KW = 32 / GP;   // keys per inner iteration
+__global__ void __launch_bounds__(kDecThreads, kDecMinCtas) decode_kernel(DecodeParams p) {
+  using L = DecLayout<D, GP>;
+  constexpr int CPL = L::CPL, R = L::R, LPK = L::LPK, KG = L::KG, N = L::N;
+  constexpr unsigned kFull = 0xffffffffu;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __nv_bfloat16* ring = reinterpret_cast<__nv_bfloat16*>(smem);  // [stage][K|V][kDecChunk][D]
   __shared__ uint64_t full[kDecStages], empty[kDecStages];
   __shared__ volatile int abort_sh;
-  __shared__ float wm[kDecWarps][GP], wl[kDecWarps][GP];
-  __shared__ float wo[kDecWarps][GP][D];
+  constexpr int kStates = kDecWarps * L::NG;  // (warp, group) partial softmax states
+  __shared__ float sm_m[kStates][GP], sm_l[kStates][GP];
+  __shared__ float sm_o[kStates][GP][D];
 
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const long long unit = blockIdx.x;
@@ -141,12 +188,13 @@ __global__ void __launch_bounds__(kDecThreads) decode_kernel(DecodeParams p) {
   }
 
   // -------------------------------------------------------------- consumers
+  const int grp = lane / LPK, sub = lane % LPK, gbase = lane & ~(LPK - 1);
   const int G = p.G;
   float qv[GP][CPL];
 #pragma unroll
   for (int h = 0; h < GP; ++h) {
     if (h < G) {
-      load_row<CPL>(p.q + ((long long)b * p.Hq + (long long)g * G + h) * D, lane, qv[h]);
+      load_slice<D, GP>(p.q + ((long long)b * p.Hq + (long long)g * G + h) * D, sub, qv[h]);
 #pragma unroll
       for (int c = 0; c < CPL; ++c) qv[h][c] *= p.scale_log2;
     } else {
@@ -159,81 +207,108 @@ __global__ void __launch_bounds__(kDecThreads) decode_kernel(DecodeParams p) {
   for (int h = 0; h < GP; ++h)
 #pragma unroll
     for (int c = 0; c < CPL; ++c) o[h][c] = 0.f;
-  float m_own = -INFINITY, l_own = 0.f;  // running max / sum of head lane % GP
+  // running max / sum of heads h0 .. h0 + R - 1 of this lane's group
+  float m_own[R], l_own[R];
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    m_own[r] = -INFINITY;
+    l_own[r] = 0.f;
+  }
+  const int kk_own = (sub * R) / GP;  // key (within the group's KG) of this lane's scores
 
   for (int i = warp; i < nc; i += kDecWarps) {
     const int st = i % kDecStages;
-    if (!__all_sync(0xffffffffu, wait_bounded(&full[st], (i / kDecStages) & 1, &abort_sh, p.err))) break;
+    if (!__all_sync(kFull, wait_bounded(&full[st], (i / kDecStages) & 1, &abort_sh, p.err))) break;
     const __nv_bfloat16* Ks = ring + (size_t)(st * 2) * kDecChunk * D;
     const __nv_bfloat16* Vs = ring + (size_t)(st * 2 + 1) * kDecChunk * D;
     const long long k0 = k_begin + (long long)i * kDecChunk;
     const int nk = (int)((k_end - k0 < kDecChunk) ? k_end - k0 : kDecChunk);
+    const bool partial = nk < kDecChunk;  // warp-uniform
 #pragma unroll 1
-    for (int kb = 0; kb < nk; kb += KW) {
-      float acc[32];
+    for (int kb = 0; kb < nk; kb += L::KEYS) {
+      const int key0 = kb + grp * KG;  // this group's first key in the chunk
+      float acc[N];
 #pragma unroll
-      for (int kk = 0; kk < KW; ++kk) {
+      for (int kk = 0; kk < KG; ++kk) {
         float kf[CPL];
-        load_row<CPL>(Ks + (size_t)(kb + kk) * D, lane, kf);  // rows past nk hold stale data: masked below
+        load_slice<D, GP>(Ks + (size_t)(key0 + kk) * D, sub, kf);  // rows past nk: stale, masked below
 #pragma unroll
         for (int h = 0; h < GP; ++h) {
-          float a = qv[h][0] * kf[0];
+          uint64_t a2 = f2_pack(0.f, 0.f);
 #pragma unroll
-          for (int c = 1; c < CPL; ++c) a = fmaf(qv[h][c], kf[c], a);
-          acc[kk * GP + h] = a;
+          for (int c = 0; c < CPL; c += 2)
+            a2 = f2_fma(f2_pack(qv[h][c], qv[h][c + 1]), f2_pack(kf[c], kf[c + 1]), a2);
+          float x0, x1;
+          f2_unpack(a2, x0, x1);
+          acc[kk * GP + h] = x0 + x1;
         }
       }
-      // butterfly: lane l ends with the sum over lanes of acc[l]
+      // reduce-scatter over the LPK lanes of the group: lane sub ends with the
+      // complete scores of pairs sub * R .. sub * R + R - 1 (key x / GP, head x % GP)
+      int cnt = N;
 #pragma unroll
-      for (int half = 16; half >= 1; half >>= 1) {
-        const bool upper = (lane & half) != 0;
+      for (int off = LPK / 2; off >= 1; off >>= 1) {
+        const bool upper = (sub & off) != 0;
+        const int half = cnt / 2;
 #pragma unroll
-        for (int e = 0; e < half; ++e) {
-          const float send = upper ? acc[e] : acc[e + half];
-          const float keep = upper ? acc[e + half] : acc[e];
-          acc[e] = keep + __shfl_xor_sync(0xffffffffu, send, half);
+        for (int e = 0; e < N / 2; ++e) {
+          if (e < half) {
+            const float send = upper ? acc[e] : acc[e + half];
+            const float keep = upper ? acc[e + half] : acc[e];
+            acc[e] = keep + __shfl_xor_sync(kFull, send, off);
+          }
         }
+        cnt = half;
       }
-      const bool key_ok = kb + lane / GP < nk;
-      const float sc = key_ok ? acc[0] : -INFINITY;
-      float mh = sc;
+      const bool key_ok = key0 + kk_own < nk;
+      float pr[R], alpha[R];
+      bool grew = false;
 #pragma unroll
-      for (int off = GP; off < 32; off <<= 1) mh = fmaxf(mh, __shfl_xor_sync(0xffffffffu, mh, off));
-      const float m_new = fmaxf(m_own, mh);
-      const float mu = (m_new == -INFINITY) ? 0.f : m_new;
-      const float pr = ex2(sc - mu);
-      const float alpha = ex2(m_own - mu);
-      float ps = pr;
+      for (int r = 0; r < R; ++r) {
+        const float sc = key_ok ? acc[r] : -INFINITY;
+        float mh = sc;
 #pragma unroll
-      for (int off = GP; off < 32; off <<= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
-      l_own = l_own * alpha + ps;
-      // O is rescaled only when some head's running max grew (alpha = 1
-      // exactly otherwise), which after the first keys is rare.
-      if (__any_sync(0xffffffffu, m_new != m_own)) {
+        for (int off = GP / R; off < LPK; off <<= 1) mh = fmaxf(mh, __shfl_xor_sync(kFull, mh, off));
+        const float m_new = fmaxf(m_own[r], mh);
+        const float mu = (m_new == -INFINITY) ? 0.f : m_new;
+        pr[r] = ex2(sc - mu);
+        alpha[r] = ex2(m_own[r] - mu);
+        float ps = pr[r];
+#pragma unroll
+        for (int off = GP / R; off < LPK; off <<= 1) ps += __shfl_xor_sync(kFull, ps, off);
+        l_own[r] = l_own[r] * alpha[r] + ps;
+        grew = grew || (m_new != m_own[r]);
+        m_own[r] = m_new;
+      }
+      // O is rescaled only when some running max grew (alpha = 1 exactly
+      // otherwise), which after the first keys is rare.
+      if (__any_sync(kFull, grew)) {
 #pragma unroll
         for (int h = 0; h < GP; ++h) {
-          const float ah = __shfl_sync(0xffffffffu, alpha, h);
+          const float ah = __shfl_sync(kFull, alpha[h % R], gbase + h / R);
 #pragma unroll
           for (int c = 0; c < CPL; ++c) o[h][c] *= ah;
         }
       }
-      m_own = m_new;
 #pragma unroll
-      for (int kk = 0; kk < KW; ++kk) {
-        if (kb + kk < nk) {  // warp-uniform
-          float vf[CPL];
-          load_row<CPL>(Vs + (size_t)(kb + kk) * D, lane, vf);
+      for (int kk = 0; kk < KG; ++kk) {
+        float vf[CPL];
+        load_slice<D, GP>(Vs + (size_t)(key0 + kk) * D, sub, vf);
+        if (partial && key0 + kk >= nk) {  // stale rows of the last chunk may hold anything
 #pragma unroll
-          for (int h = 0; h < GP; ++h) {
-            const float pk = __shfl_sync(0xffffffffu, pr, kk * GP + h);
-            const uint64_t pk2 = f2_pack(pk, pk);
+          for (int c = 0; c < CPL; ++c) vf[c] = 0.f;
+        }
 #pragma unroll
-            for (int c = 0; c < CPL; c += 2) {
-              float lo, hi;
-              f2_unpack(f2_fma(pk2, f2_pack(vf[c], vf[c + 1]), f2_pack(o[h][c], o[h][c + 1])), lo, hi);
-              o[h][c] = lo;
-              o[h][c + 1] = hi;
-            }
+        for (int h = 0; h < GP; ++h) {
+          const int x = kk * GP + h;
+          const float pk = __shfl_sync(kFull, pr[x % R], gbase + x / R);
+          const uint64_t pk2 = f2_pack(pk, pk);
+#pragma unroll
+          for (int c = 0; c < CPL; c += 2) {
+            float lo, hi;
+            f2_unpack(f2_fma(pk2, f2_pack(vf[c], vf[c + 1]), f2_pack(o[h][c], o[h][c + 1])), lo, hi);
+            o[h][c] = lo;
+            o[h][c + 1] = hi;
           }
         }
       }
@@ -242,29 +317,33 @@ __global__ void __launch_bounds__(kDecThreads) decode_kernel(DecodeParams p) {
     if (lane == 0) mbar_arrive(&empty[st]);
   }
 
-  // merge the four warps' states, then write this split's partial
-  if (lane < GP) {
-    wm[warp][lane] = m_own;
-    wl[warp][lane] = l_own;
+  // merge the (warp, group) states, then write this split's partial
+  const int state = warp * L::NG + grp;
+  if (sub < GP / R) {
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      sm_m[state][sub * R + r] = m_own[r];
+      sm_l[state][sub * R + r] = l_own[r];
+    }
   }
 #pragma unroll
   for (int h = 0; h < GP; ++h)
 #pragma unroll
-    for (int c = 0; c < CPL; ++c) wo[warp][h][lane * CPL + c] = o[h][c];
+    for (int t = 0; t < L::T; ++t)
+#pragma unroll
+      for (int e = 0; e < L::PS; ++e) sm_o[state][h][(sub + LPK * t) * L::PS + e] = o[h][t * L::PS + e];
   asm volatile("bar.sync 1, %0;" ::"n"(kDecWarps * 32) : "memory");
   float* part = p.part + (size_t)unit * G * (D + 2);
   for (int idx = threadIdx.x; idx < G * D; idx += kDecWarps * 32) {
     const int h = idx / D, c = idx % D;
     float M = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < kDecWarps; ++w) M = fmaxf(M, wm[w][h]);
+    for (int w = 0; w < kStates; ++w) M = fmaxf(M, sm_m[w][h]);
     const float Mu = (M == -INFINITY) ? 0.f : M;
     float acc = 0.f, lsum = 0.f;
-#pragma unroll
-    for (int w = 0; w < kDecWarps; ++w) {
-      const float f = ex2(wm[w][h] - Mu);
-      acc = fmaf(wo[w][h][c], f, acc);
-      lsum = fmaf(wl[w][h], f, lsum);
+    for (int w = 0; w < kStates; ++w) {
+      const float f = ex2(sm_m[w][h] - Mu);
+      acc = fmaf(sm_o[w][h][c], f, acc);
+      lsum = fmaf(sm_l[w][h], f, lsum);
     }
     part[h * (D + 2) + c] = acc;
     if (c == 0) {
