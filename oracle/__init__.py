@@ -10,7 +10,7 @@ Two independent statements of the method live here:
   (sampled rows k*gamma), Alg. 1 / Eq. 6 (Delta correction), Eq. 5
   ("recompute"), the appendix dense tail block and the appendix Delta
   smoothing (linear interpolation, EMA, Alg. 2's alpha-beta-gamma filter)
-  and Eq. 2 decoding over the cache, all in double precision.
+  Eq. 2 decoding over the cache and RoPE on Q and K, all in double precision.
 * ``brute.py``: whole-matrix numpy evaluation (explicit N x N score matrix,
   -inf masks, matrix softmax, ``np.repeat`` of Delta) for small N.
 
@@ -56,6 +56,10 @@ def _load(path=None):
         lib.oracle_decode.argtypes = [u16p, u16p, u16p, ci, ci, ci, i64, ci, ctypes.POINTER(ctypes.c_int64), dp, dp,
                                       ci]
         lib.oracle_decode.restype = ci
+        lib.oracle_rope_f64.argtypes = [u16p, i64, i64, ci, i64, ctypes.c_double, dp]
+        lib.oracle_rope_f64.restype = ci
+        lib.oracle_rope_bf16.argtypes = [u16p, i64, i64, ci, i64, ctypes.c_double, u16p]
+        lib.oracle_rope_bf16.restype = ci
         _libs[path] = lib
     return _libs[path]
 
@@ -176,6 +180,26 @@ def decode(q, K, V, n_keys, nthreads=0, lib=None):
     if rc != 0:
         raise ValueError("oracle_decode failed (invalid arguments)")
     return out, dev.value
+
+
+def rope(X, base, pos0=0, rounded=True, lib=None):
+    """RoPE (rotate-half, angle pos * base^(-2c/d)) of X [..., N, d] bf16 bits,
+    row n at position pos0 + n.  rounded=True returns bf16 bits (RNE),
+    otherwise the float64 rotation."""
+    X = _u16(X)
+    N, d = X.shape[-2], X.shape[-1]
+    rows_total = X.size // d
+    if rounded:
+        out = np.empty(X.shape, np.uint16)
+        rc = _load(lib).oracle_rope_bf16(_ptr(X, ctypes.c_uint16), rows_total, N, d, pos0, base,
+                                         _ptr(out, ctypes.c_uint16))
+    else:
+        out = np.empty(X.shape, np.float64)
+        rc = _load(lib).oracle_rope_f64(_ptr(X, ctypes.c_uint16), rows_total, N, d, pos0, base,
+                                        _ptr(out, ctypes.c_double))
+    if rc != 0:
+        raise ValueError("oracle rope failed (invalid arguments)")
+    return out
 
 
 def rows(Q, K, V, n_sink, window, gamma, bhi, nthreads=0, lib=None):

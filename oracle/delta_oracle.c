@@ -31,6 +31,9 @@
  *     added to the sparse rows.
  *   - Eq. 2: decoding after the prefill, one new query per sequence attending
  *     densely over the cached keys with its own key appended.
+ *   - Sec. 2 (positional encodings applied to Q and K before Eq. 1): RoPE in
+ *     the rotate-half form, channel c paired with c + d/2, angle
+ *     pos * base^(-2c/d).
  *
  * Readings of the paper used here (each also listed in the design notes):
  *   - Rows are 0-based and the sample for row i is row floor(i/gamma)*gamma,
@@ -742,5 +745,71 @@ int oracle_decode(const uint16_t *q, const uint16_t *K, const uint16_t *V, int B
     double dev = 0.0;
     int rc = run_pool(decode_item, &c, (int64_t)B * Hq, L, d, nthreads, &dev);
     if (max_dev) *max_dev = dev;
+    return rc;
+}
+
+/* ------------------------------------------------------------------------ */
+/* RoPE (Sec. 2: positional encodings applied to Q and K before attention).  */
+/* Rotate-half form: for c < d/2 the pair (x_c, x_{c+d/2}) at position pos   */
+/* is rotated by the angle pos * base^(-2c/d):                               */
+/*   x'_c       = x_c cos - x_{c+d/2} sin                                    */
+/*   x'_{c+d/2} = x_{c+d/2} cos + x_c sin                                    */
+/* Row r of X [rows_total = B*H*N, d] has position pos0 + (r mod N).         */
+
+static double rope_angle(int64_t pos, int c, int d, double base)
+{
+    return (double)pos * pow(base, -2.0 * (double)c / (double)d);
+}
+
+/* fp64 result (no rounding): out [B*H*N, d] doubles. */
+int oracle_rope_f64(const uint16_t *X, int64_t rows_total, int64_t N, int d, int64_t pos0, double base,
+                    double *out)
+{
+    if (!X || !out || rows_total < 1 || N < 1 || d < 2 || (d & 1) || base <= 0.0) return -1;
+    const int h = d / 2;
+    for (int64_t r = 0; r < rows_total; ++r) {
+        const int64_t pos = pos0 + r % N;
+        const uint16_t *x = X + r * d;
+        double *o = out + r * d;
+        for (int c = 0; c < h; ++c) {
+            const double a = rope_angle(pos, c, d, base);
+            const double ca = cos(a), sa = sin(a);
+            const double x0 = bf16_to_double(x[c]), x1 = bf16_to_double(x[c + h]);
+            const double sg = MUTANT(13) ? -1.0 : 1.0;
+            o[c] = x0 * ca - sg * x1 * sa;
+            o[c + h] = x1 * ca + sg * x0 * sa;
+        }
+    }
+    return 0;
+}
+
+/* double -> bf16 bits, rounded once to the nearest 8-significant-bit value,
+ * ties to even (the rotated values enter the attention as bf16, as the
+ * unrotated inputs do).  For the normal range of bf16. */
+static uint16_t double_to_bf16(double v)
+{
+    if (v == 0.0) return signbit(v) ? 0x8000u : 0u;
+    int e;
+    const double m = frexp(v, &e);                 /* v = m 2^e, 0.5 <= |m| < 1 */
+    const double r = nearbyint(ldexp(m, 8));       /* 8 significant bits, ties to even */
+    const float f = (float)ldexp(r, e - 8);        /* exact: 8 bits fit a float */
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    return (uint16_t)(u >> 16);
+}
+
+/* bf16 result: out bits [B*H*N, d]. */
+int oracle_rope_bf16(const uint16_t *X, int64_t rows_total, int64_t N, int d, int64_t pos0, double base,
+                     uint16_t *out)
+{
+    if (!out) return -1;
+    double *tmp = (double *)malloc(sizeof(double) * (size_t)d);
+    if (!tmp) return -1;
+    int rc = 0;
+    for (int64_t r = 0; r < rows_total && rc == 0; ++r) {
+        rc = oracle_rope_f64(X + r * d, 1, 1, d, pos0 + r % N, base, tmp);
+        for (int c = 0; c < d && rc == 0; ++c) out[r * d + c] = double_to_bf16(tmp[c]);
+    }
+    free(tmp);
     return rc;
 }

@@ -19,6 +19,8 @@ What pins what:
   * whole-matrix restatement -> the numpy brute force (oracle/brute.py).
   * Eq. 2 decoding           -> the dense causal row at the token's position
                                 and torch scaled_dot_product_attention.
+  * RoPE                     -> identity at position 0, the unit-vector closed
+                                form, pair norms, relative-position scores.
   * Delta smoothing          -> reductions to Eq. 6 (EMA beta = 1, filter
     (appendix Interpolation,    (1, 0, 0), linear at gamma = 1), fixed points
      Alg. 2)                    of a constant Delta, the EMA step response,
@@ -363,10 +365,43 @@ def pin_decode(lib=None):
             assert np.abs(out[b] - ref).max() <= TOL
 
 
+def pin_rope(lib=None):
+    """RoPE: position 0 is the identity; a unit vector on channel c rotates into
+    (cos a, sin a) on channels (c, c + d/2) with a = pos base^(-2c/d) (the
+    pairing and the sign); each pair keeps its norm; and the score of two
+    rotated vectors depends only on the difference of their positions."""
+    d, base = 16, 10000.0
+    X = rand_bits(70, (1, 1, 5, d))
+    assert np.array_equal(oracle.rope(X[:, :, :1], base, 0, lib=lib), X[:, :, :1])
+    for c in (0, 3, 7):
+        for pos in (1, 5, 123):
+            e = np.zeros((1, 1, 1, d), np.float32)
+            e[..., c] = 1.0
+            eb = torch.from_numpy(e).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+            r = oracle.rope(eb, base, pos, rounded=False, lib=lib)[0, 0, 0]
+            a = pos * base ** (-2.0 * c / d)
+            want = np.zeros(d)
+            want[c], want[c + d // 2] = np.cos(a), np.sin(a)
+            assert np.abs(r - want).max() <= 1e-12, (c, pos)
+    r = oracle.rope(X, base, 37, rounded=False, lib=lib)[0, 0]
+    x = f64(X)[0, 0]
+    assert np.abs(r[:, :d // 2] ** 2 + r[:, d // 2:] ** 2 - x[:, :d // 2] ** 2 - x[:, d // 2:] ** 2).max() <= 1e-12
+    q, k = rand_bits(71, (1, 1, 1, d)), rand_bits(72, (1, 1, 1, d))
+    for (m, n) in ((10, 3), (1000, 993), (50007, 50000)):
+        s = np.dot(oracle.rope(q, base, m, rounded=False, lib=lib).ravel(),
+                   oracle.rope(k, base, n, rounded=False, lib=lib).ravel())
+        s0 = np.dot(oracle.rope(q, base, 7, rounded=False, lib=lib).ravel(),
+                    oracle.rope(k, base, 0, rounded=False, lib=lib).ravel())
+        assert abs(s - s0) <= 1e-9, (m, n)
+    rb = oracle.rope(X, base, 37, lib=lib)
+    rt = torch.from_numpy(r.astype(np.float32)).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.abs(f64(rb)[0, 0] - f64(rt)).max() <= 2.0 ** -7 * np.abs(r).max()
+
+
 ALL_PINS = [pin_gamma1_is_sdpa, pin_full_window_is_sdpa, pin_zero_keys_closed_form,
             pin_window1_no_sink, pin_constant_values, pin_mask_structure,
             pin_sampled_rows_are_dense, pin_gqa_repeat, pin_lemma1, pin_rows_agree,
-            pin_smooth_reductions, pin_smooth_closed_forms, pin_decode]
+            pin_smooth_reductions, pin_smooth_closed_forms, pin_decode, pin_rope]
 # The brute-force restatements are listed separately: the mutant test shows the
 # other pins catch every planted mistake without them.
 BRUTE_PINS = [pin_brute_force, pin_smooth_brute]

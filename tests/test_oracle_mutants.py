@@ -7,7 +7,7 @@ over the sparse set, Delta taken against the current row instead of the
 sample, a transposed K operand, and three smoothing slips (EMA weights
 swapped, the filter's velocity gain replaced by its position gain, the
 interpolation weight one row ahead), and a decode that leaves out the new
-token's own key.  All of this runs on the CPU.
+token's own key, and a RoPE rotation in the wrong direction.  All of this runs on the CPU.
 """
 import os
 import tempfile
@@ -30,6 +30,7 @@ MUTANTS = {
     10: "filter velocity corrected with alpha",
     11: "linear interpolation weight one row ahead",
     12: "decode without the new token's own key",
+    13: "RoPE rotation in the wrong direction",
 }
 
 _tmp = tempfile.mkdtemp(prefix="oracle_mutants_")
