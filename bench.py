@@ -274,9 +274,37 @@ def time_variants(args, w, q, k, v, out, stream, restore):
                      "tokens_per_s": w.B * w.N / (ms / 1e3),
                      "tail_dense_pairs_per_head": flops.tail_pairs_per_head(w.N, tail)}
         del ws
+    res["rope_prefill"] = time_rope_prefill(w, q, k, v, out, stream)
     res["decode"] = time_decode(w, q, k, v, stream)
     restore()  # `out` back to the Delta result for the spot check
     return res
+
+
+def time_rope_prefill(w, q, k, v, out, stream):
+    """The prefill with RoPE fused (delta_attn_prefill_rope): K rotated in
+    place by a pass of its own, each Q tile rotated on its way into tensor
+    memory.  Timed on a copy of K, restored before every call, outside the
+    timed region."""
+    from paper_2505_11254_gb300 import binding
+    table = binding.rope_table(w.N, w.d, 500000.0, device=q.device)
+    kc = torch.empty_like(k)
+    ws = binding.alloc_workspace(binding.workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, w.gamma),
+                                 q.device)
+    times = []
+    for it in range(13):
+        kc.copy_(k)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        binding.delta_attn_prefill_rope(q, kc, v, w.n_sink, w.window, w.gamma, table, out=out, workspace=ws)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if it >= 3:
+            times.append(e0.elapsed_time(e1))
+    if binding.check() != binding.DA_OK:
+        raise RuntimeError("device status after the RoPE prefill timing")
+    ms = statistics.median(times)
+    return {"ms": ms, "tokens_per_s": w.B * w.N / (ms / 1e3), "rope_base": 500000.0,
+            "note": "K rotated in place (one pass), Q rotated inside the attention kernels"}
 
 
 def time_decode(w, q, k, v, stream):

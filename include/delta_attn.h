@@ -211,6 +211,33 @@ int delta_attn_decode_workspace_size(int B, int Hq, int Hkv, int64_t max_keys, i
 int delta_attn_decode(const void* q, const void* K, const void* V, const int64_t* lens, void* O, int B, int Hq,
                       int Hkv, int64_t L, int64_t max_keys, int d, void* workspace, size_t ws_bytes, void* stream);
 
+/* RoPE (Sec. 2: positional encodings on Q and K before the attention), in the
+ * rotate-half form: for c < d/2 the pair (x_c, x_{c+d/2}) of a row at
+ * position pos is rotated by the angle pos * base^(-2c/d).
+ *
+ * delta_attn_rope_table: writes the (cos, sin) table for positions
+ * 0 .. n_pos-1, table [n_pos][d/2][2] fp32 (device, 16-byte aligned,
+ * n_pos * d * 4 bytes), angles and sines taken in double.  Built once per
+ * (n_pos, d, base) and shared by every layer and call. */
+int delta_attn_rope_table(int64_t n_pos, int d, double base, float* table, void* stream);
+
+/* Rotates X [B, H, N, d] bf16 (device, 16-byte aligned) in place, row n at
+ * position pos0 + n (a new token's query or key at its position, or a whole
+ * K before the prefill); fp32 arithmetic, one rounding to bf16 (RNE).  The
+ * table (table_rows positions) must cover pos0 + N - 1. */
+int delta_attn_rope_apply(void* X, int B, int H, int64_t N, int d, int64_t pos0, const float* table,
+                          int64_t table_rows, void* stream);
+
+/* delta_attn_prefill() for unrotated Q and K, with RoPE fused: K is rotated
+ * in place first (on return it holds RoPE(K), the form the cache keeps for
+ * decoding), and each Q tile is rotated by the attention kernels while it is
+ * copied into tensor memory (Q itself is not modified), so no rotated copy of
+ * Q is written or read.  Positions are the row indices 0 .. N-1; the table
+ * must cover them (table_rows >= N).  Everything else as delta_attn_prefill(). */
+int delta_attn_prefill_rope(const void* Q, void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N, int d,
+                            int n_sink, int64_t window, int gamma, const float* table, int64_t table_rows,
+                            void* workspace, size_t ws_bytes, void* stream);
+
 /* Synchronises `stream`, returns and clears the device status word
  * (DA_OK, DA_ERR_TIMEOUT), or DA_ERR_CUDA if the stream reports an error. */
 int delta_attn_check(void* stream);

@@ -50,6 +50,9 @@ _SIGNATURES = {
     "delta_apply": ([_p, _p, _p, _p, _i, _i, _i64, _i, _i, _p], _i),
     "delta_attn_decode_workspace_size": ([_i, _i, _i, _i64, _i, ctypes.POINTER(_sz)], _i),
     "delta_attn_decode": ([_p, _p, _p, _p, _p, _i, _i, _i, _i64, _i64, _i, _p, _sz, _p], _i),
+    "delta_attn_rope_table": ([_i64, _i, ctypes.c_double, _p, _p], _i),
+    "delta_attn_rope_apply": ([_p, _i, _i, _i64, _i, _i64, _p, _i64, _p], _i),
+    "delta_attn_prefill_rope": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _i64, _p, _sz, _p], _i),
     "delta_attn_check": ([_p], _i),
     "delta_attn_status_string": ([_i], ctypes.c_char_p),
     "delta_attn_plan_info": ([_i, _i, _i, _i64, _i, _i, _i64, _i, ctypes.POINTER(_i64)], _i),
@@ -216,6 +219,35 @@ def decode(q, k_cache, v_cache, lens=None, max_keys=None, out=None, workspace=No
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     _check(load().delta_attn_decode(_dptr(q), _dptr(k_cache), _dptr(v_cache), _dptr(lens), _dptr(out), B, Hq, Hkv,
                                     L, max_keys, d, _dptr(workspace), ws_bytes, _stream(stream)), "delta_attn_decode")
+    return out
+
+
+def rope_table(n_pos, d, base, device="cuda", stream=None):
+    """RoPE (cos, sin) table fp32 [n_pos, d/2, 2] for positions 0..n_pos-1."""
+    t = torch.empty((n_pos, d // 2, 2), dtype=torch.float32, device=device)
+    _check(load().delta_attn_rope_table(n_pos, d, float(base), _dptr(t), _stream(stream)), "delta_attn_rope_table")
+    return t
+
+
+def rope_apply(x, table, pos0=0, stream=None):
+    """Rotates x [B,H,N,d] bf16 in place (row n at position pos0 + n)."""
+    if x.dim() != 4 or x.dtype != torch.bfloat16 or not x.is_cuda or not x.is_contiguous():
+        raise ValueError("x: contiguous bf16 CUDA tensor [B,H,N,d]")
+    B, H, N, d = x.shape
+    _check(load().delta_attn_rope_apply(_dptr(x), B, H, N, d, pos0, _dptr(table), table.shape[0], _stream(stream)),
+           "delta_attn_rope_apply")
+    return x
+
+
+def delta_attn_prefill_rope(q, k, v, n_sink, window, gamma, table, out=None, workspace=None, stream=None):
+    """The prefill for unrotated q and k with RoPE fused (k rotated in place)."""
+    B, Hq, Hkv, N, d = _qkv_shape(q, k, v)
+    if out is None:
+        out = torch.empty_like(q)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(load().delta_attn_prefill_rope(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink,
+                                          window, gamma, _dptr(table), table.shape[0], _dptr(workspace), ws_bytes,
+                                          _stream(stream)), "delta_attn_prefill_rope")
     return out
 
 

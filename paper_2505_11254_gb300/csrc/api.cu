@@ -401,15 +401,20 @@ int delta_attn_plan_info(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, i
   return DA_OK;
 }
 
+// rope: a (cos, sin) table [>= N][d/2][2] when Q and K come unrotated; K is
+// then rotated in place before the first kernel and every Q tile on its way
+// into tensor memory.
 static int prefill_impl(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
                         int d, int n_sink, int64_t window, int gamma, int mode, int64_t tail, const SmoothArgs& sm,
-                        void* workspace, size_t ws_bytes, void* stream, void* const* events, int n_events) {
+                        void* workspace, size_t ws_bytes, void* stream, void* const* events, int n_events,
+                        const float* rope = nullptr) {
   if (!Q || !K || !V || !O) return DA_ERR_INVALID_ARG;
   int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
   if (rc) return rc;
   if ((rc = check_variant(mode, tail, N))) return rc;
   if ((rc = check_smooth(sm, mode))) return rc;
-  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(workspace))
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O) || !aligned16(workspace) ||
+      !aligned16(rope))
     return DA_ERR_MISALIGNED;
   int sms = 0;
   if ((rc = check_device(&sms))) return rc;
@@ -428,6 +433,11 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
 
   ScopedWorkspace ws(workspace, pl.total, s);
   if (ws.failed()) return DA_ERR_CUDA;
+  if (rope != nullptr) {
+    if (launch_rope_apply(const_cast<void*>(K), (long long)B * Hkv * N, N, d, 0, rope, s) != cudaSuccess)
+      return DA_ERR_CUDA;
+    p.rope = rope;
+  }
   uint8_t* base = ws.get();
   p.partials = reinterpret_cast<float*>(base + pl.off_part);
   p.counter = reinterpret_cast<unsigned long long*>(base + pl.off_ticket);
@@ -436,6 +446,7 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   Params pt = pl.pt;
   if (pl.tail > 0) {
     pt.err = p.err;
+    pt.rope = p.rope;
     pt.partials = reinterpret_cast<float*>(base + pl.off_tail_part);
     pt.counter = reinterpret_cast<unsigned long long*>(base + pl.off_tail_ticket);
     pt.tickets = reinterpret_cast<int*>(base + pl.off_tail_ticket + 4 * sizeof(unsigned long long));
@@ -661,6 +672,36 @@ int delta_attn_decode(const void* q, const void* K, const void* V, const int64_t
   p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
   p.part = reinterpret_cast<float*>(ws.get());
   return launch_decode(p, O, s) == cudaSuccess ? DA_OK : DA_ERR_CUDA;
+}
+
+int delta_attn_rope_table(int64_t n_pos, int d, double base, float* table, void* stream) {
+  if (!table || n_pos < 1 || n_pos > (int64_t(1) << 34) || !(base > 0.0) || !std::isfinite(base))
+    return DA_ERR_INVALID_ARG;
+  if (d != 64 && d != 128) return DA_ERR_UNSUPPORTED;
+  if (!aligned16(table)) return DA_ERR_MISALIGNED;
+  return launch_rope_table(n_pos, d, base, table, static_cast<cudaStream_t>(stream)) == cudaSuccess ? DA_OK
+                                                                                                  : DA_ERR_CUDA;
+}
+
+int delta_attn_rope_apply(void* X, int B, int H, int64_t N, int d, int64_t pos0, const float* table,
+                          int64_t table_rows, void* stream) {
+  if (!X || !table || B < 1 || H < 1 || N < 1 || pos0 < 0 || (int64_t)B * H > (int64_t(1) << 30))
+    return DA_ERR_INVALID_ARG;
+  if (d != 64 && d != 128) return DA_ERR_UNSUPPORTED;
+  if (pos0 + N > table_rows) return DA_ERR_INVALID_ARG;  // the table must cover every position
+  if (!aligned16(X) || !aligned16(table)) return DA_ERR_MISALIGNED;
+  return launch_rope_apply(X, (long long)B * H * N, N, d, pos0, table, static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? DA_OK
+             : DA_ERR_CUDA;
+}
+
+int delta_attn_prefill_rope(const void* Q, void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N, int d,
+                            int n_sink, int64_t window, int gamma, const float* table, int64_t table_rows,
+                            void* workspace, size_t ws_bytes, void* stream) {
+  if (!table || table_rows < N) return DA_ERR_INVALID_ARG;
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, DA_MODE_DELTA, 0, SmoothArgs{},
+                      workspace, ws_bytes, stream, nullptr, 0, table);
 }
 
 int delta_attn_check(void* stream) {

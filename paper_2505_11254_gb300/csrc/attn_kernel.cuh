@@ -551,7 +551,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int nq = 0;
     // Q of an item: swizzled smem rows -> TMEM lanes (bf16 pairs), the A
     // operand of S = Q K^T.
-    auto copy_q = [&](int buf) {
+    auto copy_q = [&](int buf, long long qitem) {
       ok = ok && __all_sync(kFull, wait_sleepy(&bars.q_full, nq & 1, &abort_sh, p.err));
       ++nq;
       if (ok) {
@@ -567,6 +567,26 @@ __global__ void __launch_bounds__(kThreads, 1)
             r[ch * 32 + pc * 4 + 2] = v.z;
             r[ch * 32 + pc * 4 + 3] = v.w;
           }
+        if (p.rope != nullptr) {
+          // RoPE (Sec. 2), rotate-half: channel c turns with channel c + D/2 by
+          // the angle of the row's position; word k of r holds channels 2k and
+          // 2k + 1, its partner word is k + D/4.  fp32, one rounding to bf16.
+          const Work wq = decode_work<MODE>(p, qitem);
+          long long qrow, qsample;
+          int qhead;
+          if (lane_row<MODE>(p, wq, e, qrow, qsample, qhead)) {
+            const float4* cs = reinterpret_cast<const float4*>(p.rope + qrow * D);
+#pragma unroll
+            for (int k = 0; k < D / 4; ++k) {
+              const float4 t = __ldg(cs + k);  // (cos, sin) of channels 2k, 2k + 1
+              const float a0 = __uint_as_float(r[k] << 16), a1 = __uint_as_float(r[k] & 0xffff0000u);
+              const float b0 = __uint_as_float(r[k + D / 4] << 16);
+              const float b1 = __uint_as_float(r[k + D / 4] & 0xffff0000u);
+              r[k] = pack_bf16x2(a0 * t.x - b0 * t.y, a1 * t.z - b1 * t.w);
+              r[k + D / 4] = pack_bf16x2(b0 * t.x + a0 * t.y, b1 * t.z + a1 * t.w);
+            }
+          }
+        }
 #pragma unroll
         for (int q = 0; q < D / 64; ++q) {
           uint32_t rr[32];
@@ -583,11 +603,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
     ItemReader<DYN, true> items{(long long)blockIdx.x};
     long long item = items.next(p, iq, &abort_sh);
-    if (item >= 0) copy_q(0);
+    if (item >= 0) copy_q(0, item);
     for (int i = 0; item >= 0; ++i) {
       const Work w = decode_work<MODE>(p, item);
       const long long nxt = items.next(p, iq, &abort_sh);
-      if (nxt >= 0) copy_q((i + 1) & 1);
+      if (nxt >= 0) copy_q((i + 1) & 1, nxt);
       long long row, sample;
       int head;
       const bool row_ok = lane_row<MODE>(p, w, e, row, sample, head);

@@ -41,6 +41,12 @@ int decode_keys_per_split();
 int decode_ctas_per_sm(int d, int G);  // resident decode CTAs per SM (occupancy)
 cudaError_t launch_decode(const DecodeParams& p, void* out, cudaStream_t s);
 
+// RoPE (rope.cu): the (cos, sin) table [n_pos][d/2] fp32 pairs, and an in-place
+// rotation of bf16 rows (row r at position pos0 + r % N).
+cudaError_t launch_rope_table(long long n_pos, int d, double base, float* table, cudaStream_t s);
+cudaError_t launch_rope_apply(void* x, long long rows, long long N, int d, long long pos0, const float* table,
+                              cudaStream_t s);
+
 cudaError_t launch_debug_mask(long long N, int n_sink, long long window, long long i0, long long i1,
                               unsigned char* out, cudaStream_t s);
 cudaError_t launch_debug_rowmap(long long N, int gamma, long long* sample_row, unsigned char* sampled,

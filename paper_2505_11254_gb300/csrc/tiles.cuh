@@ -72,6 +72,7 @@ struct Params {
   float* delta_out;        // [B,Hq,n_s,d] fp32
   const float* smooth_basis;  // [B,Hq,n_s,kSmoothJ,d] fp32 (EPI_FUSED_SMOOTH)
   const float* smooth_coef;   // [gamma][kSmoothJ] fp32 (EPI_FUSED_SMOOTH)
+  const float* rope;          // RoPE (cos, sin) table [N][d/2][2] fp32: Q rotated on its way to TMEM, or null
   float* partials;         // n_multi slots of BM*(d+2) fp32
   int* tickets;            // n_multi
   unsigned long long* counter;  // dynamic item counter (zeroed before the launch)
