@@ -238,6 +238,27 @@ int delta_attn_prefill_rope(const void* Q, void* K, const void* V, void* O, int 
                             int n_sink, int64_t window, int gamma, const float* table, int64_t table_rows,
                             void* workspace, size_t ws_bytes, void* stream);
 
+/* Workspace bytes delta_attn_prefill_host() needs: two device staging buffers
+ * of one (batch, KV head) chunk (its G query heads of Q and O, one K and V
+ * head) and the workspace of a chunk's prefill.  Returns a da_status. */
+int delta_attn_host_workspace_size(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma,
+                                   size_t* bytes);
+
+/* delta_attn_prefill() on HOST buffers: Qh, Kh, Vh, Oh with the layouts of
+ * delta_attn_prefill() in host memory (page-locked for asynchronous copies).
+ * The B * Hkv (batch, KV head) chunks are independent, so their copies in,
+ * prefills and copies out are pipelined over three streams (two internal copy
+ * streams, created once per device, and `stream` for the kernels), with two
+ * device staging buffers in the workspace (device, 256-byte aligned, or NULL
+ * for stream-ordered allocation on `stream`).  Asynchronous: Oh is complete
+ * when `stream` reaches the end of the call.  Each chunk's prefill is
+ * delta_attn_prefill() with B = 1, Hq = G, Hkv = 1 (the split-K plan of the
+ * dense rows follows the chunk's size, so the result may differ from one
+ * whole-problem call in the last bits of fp32 rounding order). */
+int delta_attn_prefill_host(const void* Qh, const void* Kh, const void* Vh, void* Oh, int B, int Hq, int Hkv,
+                            int64_t N, int d, int n_sink, int64_t window, int gamma, void* workspace,
+                            size_t ws_bytes, void* stream);
+
 /* Synchronises `stream`, returns and clears the device status word
  * (DA_OK, DA_ERR_TIMEOUT), or DA_ERR_CUDA if the stream reports an error. */
 int delta_attn_check(void* stream);

@@ -53,6 +53,8 @@ _SIGNATURES = {
     "delta_attn_rope_table": ([_i64, _i, ctypes.c_double, _p, _p], _i),
     "delta_attn_rope_apply": ([_p, _i, _i, _i64, _i, _i64, _p, _i64, _p], _i),
     "delta_attn_prefill_rope": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _i64, _p, _sz, _p], _i),
+    "delta_attn_host_workspace_size": ([_i, _i, _i, _i64, _i, _i, _i64, _i, ctypes.POINTER(_sz)], _i),
+    "delta_attn_prefill_host": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _sz, _p], _i),
     "delta_attn_check": ([_p], _i),
     "delta_attn_status_string": ([_i], ctypes.c_char_p),
     "delta_attn_plan_info": ([_i, _i, _i, _i64, _i, _i, _i64, _i, ctypes.POINTER(_i64)], _i),
@@ -248,6 +250,31 @@ def delta_attn_prefill_rope(q, k, v, n_sink, window, gamma, table, out=None, wor
     _check(load().delta_attn_prefill_rope(_dptr(q), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N, d, n_sink,
                                           window, gamma, _dptr(table), table.shape[0], _dptr(workspace), ws_bytes,
                                           _stream(stream)), "delta_attn_prefill_rope")
+    return out
+
+
+def host_workspace_size(B, Hq, Hkv, N, d, n_sink, window, gamma) -> int:
+    out = _sz(0)
+    _check(load().delta_attn_host_workspace_size(B, Hq, Hkv, N, d, n_sink, window, gamma, ctypes.byref(out)),
+           "delta_attn_host_workspace_size")
+    return out.value
+
+
+def delta_attn_prefill_host(qh, kh, vh, n_sink, window, gamma, out=None, workspace=None, stream=None):
+    """The prefill on host tensors (bf16, contiguous, page-locked): copies in,
+    kernels and copies out pipelined per (batch, KV head) chunk.  Returns the
+    host output tensor; it is complete once the stream reaches this point."""
+    for name, t in (("q", qh), ("k", kh), ("v", vh)):
+        if t.dtype != torch.bfloat16 or t.is_cuda or not t.is_contiguous() or t.dim() != 4:
+            raise ValueError("%s: contiguous bf16 host tensor [B,H,N,d]" % name)
+    B, Hq, N, d = qh.shape
+    Hkv = kh.shape[1]
+    if out is None:
+        out = torch.empty(qh.shape, dtype=torch.bfloat16, pin_memory=True)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(load().delta_attn_prefill_host(_dptr(qh), _dptr(kh), _dptr(vh), _dptr(out), B, Hq, Hkv, N, d, n_sink,
+                                          window, gamma, _dptr(workspace), ws_bytes, _stream(stream)),
+           "delta_attn_prefill_host")
     return out
 
 
