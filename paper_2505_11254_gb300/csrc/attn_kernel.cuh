@@ -430,6 +430,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       long long row, sample;
       int head;
       lane_row<MODE>(p, w, t, row, sample, head);
+      int j_plain0, j_plain1;  // tiles [j_plain0, j_plain1) need no mask
+      unmasked_tiles<MODE>(p, w, j_plain0, j_plain1);
       float m_run = -INFINITY, l_run = 0.f;
       for (int j = 0; ok && j < w.T; ++j, ++g) {
         if (!__all_sync(kFull, wait_bounded(&bars.s_full[g & 1], (g >> 1) & 1, &abort_sh, p.err))) {
@@ -442,7 +444,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sb = C::COL_S + (uint32_t)(g & 1) * BN;
         float s[BN];
         tmem_ld_row<BN>(tmem + la + sb, s);
-        if (tile_needs_mask<MODE>(p, w, j)) {
+        if (j < j_plain0 || j >= j_plain1) {
           // Visible key offsets c of this tile: lo <= c <= hi (window and
           // causality), plus c < se (sinks).  Branch-free selects; the sink
           // term only in tiles that hold sink keys.

@@ -224,6 +224,28 @@ __host__ __device__ __forceinline__ bool tile_needs_mask(const Params& p, const 
   }
 }
 
+// Floor division (the truncating / of C++ rounds negative quotients up).
+__host__ __device__ __forceinline__ long long floor_div(long long a, long long b) {
+  return a >= 0 ? a / b : -((-a + b - 1) / b);
+}
+
+// The item's tiles j0 <= j < j1 are exactly the ones tile_needs_mask() rejects:
+// band tiles whose every key is visible to every row of the item (causal bound
+// kt*BN + BN-1 <= first row, window bound kt*BN > last row - window).  Sink
+// tiles are never in the range.  Evaluated once per item, so the per-tile test
+// is two integer compares.
+template <int MODE>
+__host__ __device__ __forceinline__ void unmasked_tiles(const Params& p, const Work& w, int& j0, int& j1) {
+  const long long rf = (MODE == MODE_SPARSE) ? w.r0
+                       : (MODE == MODE_STRIDED_DENSE) ? p.row0 + w.r0 * p.gamma : w.r0 * p.gamma;
+  const long long rl = (MODE == MODE_SPARSE) ? w.r_last : w.r_last * p.gamma;
+  const long long k_causal = floor_div(rf - (BN - 1), BN);  // last tile all rows see causally
+  const long long k_window = (MODE == MODE_STRIDED_DENSE) ? w.kt_lo : floor_div(rl - p.window, BN) + 1;
+  const long long lo = lmax(w.kt_lo, k_window), hi = lmin(w.kt_hi, k_causal);
+  j0 = w.n_sink_tiles + (int)(lo - w.kt_lo);
+  j1 = hi >= lo ? w.n_sink_tiles + (int)(hi - w.kt_lo) + 1 : j0;
+}
+
 // Query row and head of TMEM lane t.  Returns false for padding lanes.
 template <int MODE>
 __host__ __device__ __forceinline__ bool lane_row(const Params& p, const Work& w, int t, long long& row,
