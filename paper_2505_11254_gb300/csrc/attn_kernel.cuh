@@ -616,7 +616,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = ok && __all_sync(kFull, wait_sleepy(&bars.l_ready[i & 1], (i >> 1) & 1, &abort_sh, p.err));
       const float l_row = lfin[i & 1][e], m_row = mfin[i & 1][e];
       mbar_arrive(&bars.l_free[i & 1]);
-      ok = ok && __all_sync(kFull, wait_sleepy(&bars.o_full, i & 1, &abort_sh, p.err));
+      // O lands about one PV after l_ready: a short wait, polled without sleeping
+      // so that the next item's first PV is not held back by a sleep interval.
+      ok = ok && __all_sync(kFull, wait_bounded(&bars.o_full, i & 1, &abort_sh, p.err));
       tc_fence_after();
       float o[D];
       tmem_ld_row<D>(tmem + la + C::COL_O, o);
