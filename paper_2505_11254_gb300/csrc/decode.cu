@@ -380,8 +380,15 @@ __global__ void __launch_bounds__(128) decode_merge_kernel(const float* __restri
 template <int D, int GP>
 cudaError_t launch_decode_t(const DecodeParams& p, long long units, cudaStream_t s) {
   auto k = decode_kernel<D, GP>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, dec_smem_bytes<D>());
+  static bool attr_set[64] = {};  // the attribute is set once per function and device
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64 || !attr_set[dev]) {
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, dec_smem_bytes<D>());
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) attr_set[dev] = true;
+  }
   k<<<(unsigned)units, kDecThreads, dec_smem_bytes<D>(), s>>>(p);
   return cudaGetLastError();
 }
