@@ -19,8 +19,9 @@
 //     log2(e)/sqrt(d) folded into q) then broadcasts each weight to the
 //     group's lanes for P.V with packed fp32 FMAs;
 //   * the (warp, group) partial states are merged in shared memory and written as
-//     (unnormalised o, max, sum) per split; a second kernel merges the splits
-//     in a fixed order (deterministic) and writes bf16.
+//     (unnormalised o, max, sum) per split; a second kernel, launched as a
+//     programmatic dependent so that its launch overlaps this one, merges the
+//     splits in a fixed order (deterministic) and writes bf16.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -153,6 +154,8 @@ __global__ void __launch_bounds__(kDecThreads, kDecMinCtas) decode_kernel(Decode
   const int nc = k_end > k_begin ? (int)((k_end - k_begin + kDecChunk - 1) / kDecChunk) : 0;
 
   if (threadIdx.x == 0) {
+    // let the merge grid be scheduled now; it waits for this grid's completion
+    asm volatile("griddepcontrol.launch_dependents;");
     for (int i = 0; i < kDecStages; ++i) {
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 1);
@@ -353,28 +356,81 @@ __global__ void __launch_bounds__(kDecThreads, kDecMinCtas) decode_kernel(Decode
   }
 }
 
-// One thread per (batch, query head, column): the splits in order.
-__global__ void __launch_bounds__(128) decode_merge_kernel(const float* __restrict__ part, __nv_bfloat16* out,
-                                                           long long rows, int Hq, int Hkv, int G, int n_split,
-                                                           int d) {
-  const long long t = blockIdx.x * (long long)blockDim.x + threadIdx.x;
-  if (t >= rows * d) return;
-  const long long bh = t / d;
-  const int c = (int)(t % d);
+// One CTA per (batch, query head): the split weights 2^(m_s - M) and the
+// weighted sum of the split sums are formed once in shared memory; then each
+// warp accumulates every column over its own residue class of splits (a lane
+// holds columns lane + 32 j, so a warp reads each split's row in 128-byte
+// pieces) and the warps' sums are added in warp order.  Every reduction has
+// a fixed shape and order, so the result does not depend on timing.
+constexpr int kMergeWarps = 8;
+constexpr int kMergeThreads = kMergeWarps * 32;
+
+__device__ __forceinline__ float block_reduce(float v, float* red, bool is_max) {
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float x = __shfl_xor_sync(0xffffffffu, v, o);
+    v = is_max ? fmaxf(v, x) : v + x;
+  }
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float r = red[0];
+#pragma unroll
+  for (int w = 1; w < kMergeWarps; ++w) r = is_max ? fmaxf(r, red[w]) : r + red[w];
+  __syncthreads();  // red is reused by the next reduction
+  return r;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kMergeThreads) decode_merge_kernel(const float* __restrict__ part,
+                                                                     __nv_bfloat16* out, int Hq, int Hkv, int G,
+                                                                     int n_split) {
+  constexpr int J = D / 32;  // columns per lane
+  extern __shared__ float w_sh[];  // [n_split] split weights
+  __shared__ float red[kMergeWarps];
+  __shared__ float acc_sh[kMergeWarps][D];
+  // The partials are written by the split kernel, which may still be running
+  // when this grid is scheduled (programmatic dependent launch): wait for it
+  // to complete and its writes to be visible.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const long long bh = blockIdx.x;
   const long long b = bh / Hq;
   const int h = (int)(bh % Hq), g = h / G, hh = h % G;
-  const float* base = part + ((size_t)(b * Hkv + g) * n_split) * G * (d + 2) + (size_t)hh * (d + 2);
-  const size_t stride = (size_t)G * (d + 2);
-  float M = -INFINITY;
-  for (int s = 0; s < n_split; ++s) M = fmaxf(M, base[s * stride + d]);
+  const float* base = part + ((size_t)(b * Hkv + g) * n_split) * G * (D + 2) + (size_t)hh * (D + 2);
+  const size_t stride = (size_t)G * (D + 2);
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+
+  float m = -INFINITY;
+  for (int s = threadIdx.x; s < n_split; s += kMergeThreads) m = fmaxf(m, base[s * stride + D]);
+  const float M = block_reduce(m, red, true);
   const float Mu = (M == -INFINITY) ? 0.f : M;
-  float acc = 0.f, lsum = 0.f;
-  for (int s = 0; s < n_split; ++s) {
-    const float f = ex2(base[s * stride + d] - Mu);
-    acc = fmaf(base[s * stride + c], f, acc);
-    lsum = fmaf(base[s * stride + d + 1], f, lsum);
+  float l = 0.f;
+  for (int s = threadIdx.x; s < n_split; s += kMergeThreads) {
+    const float f = ex2(base[s * stride + D] - Mu);
+    w_sh[s] = f;
+    l = fmaf(base[s * stride + D + 1], f, l);
   }
-  out[t] = __float2bfloat16_rn(lsum > 0.f ? acc / lsum : 0.f);
+  const float lsum = block_reduce(l, red, false);  // its barriers also publish w_sh
+
+  float a[J];
+#pragma unroll
+  for (int j = 0; j < J; ++j) a[j] = 0.f;
+#pragma unroll 4
+  for (int s = warp; s < n_split; s += kMergeWarps) {
+    const float f = w_sh[s];
+    const float* row = base + s * stride + lane;
+#pragma unroll
+    for (int j = 0; j < J; ++j) a[j] = fmaf(row[32 * j], f, a[j]);
+  }
+#pragma unroll
+  for (int j = 0; j < J; ++j) acc_sh[warp][lane + 32 * j] = a[j];
+  __syncthreads();
+  if (threadIdx.x < D) {
+    float acc = 0.f;
+#pragma unroll
+    for (int w = 0; w < kMergeWarps; ++w) acc += acc_sh[w][threadIdx.x];
+    out[bh * D + threadIdx.x] = __float2bfloat16_rn(lsum > 0.f ? acc / lsum : 0.f);
+  }
 }
 
 template <int D, int GP>
@@ -435,13 +491,30 @@ int decode_ctas_per_sm(int d, int G) { return d == 64 ? ctas_per_sm_d<64>(G) : c
 
 cudaError_t launch_decode(const DecodeParams& p, void* out, cudaStream_t s) {
   const long long units = (long long)p.B * p.Hkv * p.n_split;
-  if (units <= 0 || units > 0x7fffffffLL) return cudaErrorInvalidValue;
+  const long long rows = (long long)p.B * p.Hq;
+  if (units <= 0 || units > 0x7fffffffLL || rows > 0x7fffffffLL) return cudaErrorInvalidValue;
+  const size_t w_bytes = (size_t)p.n_split * sizeof(float);
+  if (w_bytes > 32768) return cudaErrorInvalidValue;  // far above one wave of splits on any GPU
   cudaError_t e = p.D == 64 ? launch_decode_d<64>(p, units, s) : launch_decode_d<128>(p, units, s);
   if (e != cudaSuccess) return e;
-  const long long rows = (long long)p.B * p.Hq;
-  const long long threads = rows * p.D;
-  decode_merge_kernel<<<(unsigned)((threads + 127) / 128), 128, 0, s>>>(
-      p.part, static_cast<__nv_bfloat16*>(out), rows, p.Hq, p.Hkv, p.G, p.n_split, p.D);
+  // The merge grid is launched as a programmatic dependent of the split
+  // kernel: it is scheduled while the split kernel runs and waits on the
+  // device (griddepcontrol.wait) for its partials.
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)rows);
+  cfg.blockDim = dim3(kMergeThreads);
+  cfg.dynamicSmemBytes = w_bytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const float* part = p.part;
+  __nv_bfloat16* o = static_cast<__nv_bfloat16*>(out);
+  e = p.D == 64 ? cudaLaunchKernelEx(&cfg, decode_merge_kernel<64>, part, o, p.Hq, p.Hkv, p.G, p.n_split)
+                : cudaLaunchKernelEx(&cfg, decode_merge_kernel<128>, part, o, p.Hq, p.Hkv, p.G, p.n_split);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

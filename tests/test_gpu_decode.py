@@ -1,7 +1,7 @@
 """Eq. 2 decoding over the cache (delta_attn_decode) against the fp64 oracle:
 GQA ratios 1 to 16 (including ratios that are not powers of two), d = 64 and
 128, per-sequence lengths shorter than the cache, a single key, lengths that
-end inside a ring chunk, and the 131K-token cache of the prefill workload
+end inside a ring chunk, hundreds of key-range splits for one head, and the 131K-token cache of the prefill workload
 with the new token's key and value appended."""
 import numpy as np
 import pytest
@@ -30,6 +30,9 @@ CASES = [
     (2, 6, 2, 333, 128, [333, 200]),
     (1, 5, 1, 128, 128, [100]),
     (4, 2, 2, 70, 64, [65, 1, 70, 63]),
+    # one (batch, KV head) pair: a wave of splits (more than the merge CTA's threads)
+    (1, 1, 1, 65536, 64, None),
+    (1, 2, 1, 40000, 128, [39999]),
 ]
 
 
