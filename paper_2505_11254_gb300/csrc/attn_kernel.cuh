@@ -10,21 +10,24 @@
 // Warp roles (384 threads = 3 warpgroups):
 //   warps 0-3  softmax: one query row per thread; S (TMEM) -> P (bf16, TMEM,
 //              aliasing S); lazy O rescaling; per item the row sum l and max m.
-//   warps 4-7  epilogue: copies the next item's Q (smem -> TMEM) ahead of time,
-//              then reads O out of TMEM, releases it, normalises, applies the
-//              Delta correction and writes the output.
-//   warp 8     TMA producer: Q of the next item, K/V tiles through a ring.
-//   warp 9     QK issuer: S = Q K^T (Q from TMEM, K from smem) once its K
-//              tile has landed and PV(g-2) has freed the S buffer.
+//   warps 4-7  epilogue: rotates the next item's Q in smem ahead of time when
+//              RoPE is on, then reads O out of TMEM, releases it, normalises,
+//              applies the Delta correction and writes the output.
+//   warp 8     TMA producer: Q of the next item, K tiles through their ring.
+//   warp 9     QK issuer: S = Q K^T (Q and K from smem) once its K tile has
+//              landed and PV(g-3) has freed the S buffer; Q is double-buffered
+//              in smem (item i in buffer i & 1).
 //   warp 10    PV issuer: O += P V (P from TMEM, V from smem) once the softmax
 //              has written P(g).  Two issuing threads keep the tensor pipe fed:
 //              neither waits on the other's inputs.
-//   warp 11    idle (it completes the third warpgroup).
+//   warp 11    V producer: V tiles through their own ring, so K loads never
+//              wait for a PV to free a slot.
 // Registers: launched at 168 per thread (384 x 168 = 64512); the third
 // warpgroup gives back to 72 and the softmax and epilogue warpgroups grow to
 // 216, so 2 x 128 x 216 + 128 x 72 = 64512 exactly.
-// TMEM (512 columns): Q double buffer [0,64) [64,128) (bf16 pairs), S/P double
-// buffer [128,256) [256,384), O [384, 384 + D).
+// TMEM (512 columns): S/P triple buffer [0,128) [128,256) [256,384), O
+// [384, 384 + D).  Three S buffers let QK run up to three tiles ahead of the
+// softmax, so the chain softmax(g) -> PV(g) -> QK(g+3) spans three tiles.
 // Every wait is bounded: past its limit a wait sets the CTA's abort flag and
 // the device status word, the roles stop working (keeping every named barrier
 // and warp-collective instruction uniform), drain their in-flight copies and
@@ -53,28 +56,42 @@ static_assert(2 * 128 * kRegsCompute + 128 * kRegsControl <= kThreads * 168, "re
 constexpr float RESCALE_THRESHOLD = 64.0f;
 constexpr uint32_t kFull = 0xffffffffu;
 
-template <int D>
+// Two TMEM layouts (512 columns):
+//   Q in TMEM (the dense pass): Q double buffer [0,64) [64,128) (bf16 pairs),
+//     S/P double buffer [128,256) [256,384), O [384, 384 + D); QK reads Q from
+//     TMEM, so a tile's shared-memory traffic is its K and V only;
+//   Q in smem (the sink + window passes): S/P triple buffer [0,128) [128,256)
+//     [256,384), O [384, 384 + D); QK reads Q and K from smem and may run
+//     three tiles ahead of the softmax.
+template <int D, int MODE = MODE_SPARSE>
 struct Cfg {
-  static constexpr int NS = (D == 128) ? 5 : 8;  // K/V ring slots (one K or V tile each)
+  static constexpr bool QTMEM = (MODE == MODE_STRIDED_DENSE);
+  static constexpr int NQ = (D == 128 || QTMEM) ? 1 : 2;  // Q buffers in smem
+  static constexpr int NK = (D == 128) ? 3 : 4;           // K ring slots (D = 128: five fit beside Q)
+  static constexpr int NV = (D == 128) ? 2 : 4;           // V ring slots
+  static constexpr int NS = NK + NV;
+  static constexpr int NSB = QTMEM ? 2 : 3;               // S/P buffers in TMEM
   static constexpr int CHUNKS = D / 64;          // 64-element (128-byte) swizzle columns
   static constexpr uint32_t Q_BYTES = BM * D * 2;
   static constexpr uint32_t KV_BYTES = BN * D * 2;
   static constexpr uint32_t SBUF_BYTES = kSampleBufBytes;  // sampled sparse rows of the fused epilogue
-  static constexpr uint32_t SMEM = Q_BYTES + NS * KV_BYTES + SBUF_BYTES + 1024;
+  static constexpr uint32_t SMEM = NQ * Q_BYTES + NS * KV_BYTES + SBUF_BYTES + 1024;
   static constexpr uint32_t TMEM_COLS = 512;
-  static constexpr uint32_t COL_Q = 0;           // + 64 * buffer
-  static constexpr uint32_t COL_S = 128;         // + BN * buffer
+  static constexpr uint32_t COL_Q = 0;                  // + 64 * buffer (Q in TMEM)
+  static constexpr uint32_t COL_S = QTMEM ? 128 : 0;    // + BN * buffer
   static constexpr uint32_t COL_O = 384;
   static constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, 0, 0);
   static constexpr uint32_t IDESC_PV = idesc_bf16(BM, D, 0, 1);
+  static_assert(COL_O + D <= TMEM_COLS, "TMEM layout");
+  static_assert(SMEM <= 232448, "shared memory above the 227 KB per-block limit");
 };
 
 struct Bars {
-  uint64_t full[8], empty[8];
-  uint64_t q_full, q_free;
+  uint64_t kfull[4], kempty[4], vfull[4], vempty[4];
+  uint64_t q_full[2], q_free[2];
   uint64_t qt_ready[2];
-  uint64_t s_full[2], p_full[2];
-  uint64_t pv_done[2], o_full, o_free;
+  uint64_t s_full[3], p_full[3];
+  uint64_t pv_done[3], o_full, o_free;
   uint64_t l_ready[2], l_free[2];
   uint64_t drain, drain2;
 };
@@ -170,7 +187,7 @@ __device__ __forceinline__ void tmem_ld_row(uint32_t addr, float (&v)[NCOL]) {
 // items from a global counter, longest first, and publishes them to the other
 // roles through a small shared-memory queue; the others read them in order.
 constexpr int kQueue = 8;
-constexpr int kQueueReaders = 10;  // QK and PV threads + 4 softmax warps + 4 epilogue warps
+constexpr int kQueueReaders = 11;  // V producer, QK and PV threads + 4 softmax warps + 4 epilogue warps
 struct ItemQueue {
   long long item[kQueue];
   uint64_t full[kQueue], empty[kQueue];
@@ -209,12 +226,13 @@ template <int D, int MODE, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const Params p) {
-  using C = Cfg<D>;
+  using C = Cfg<D, MODE>;
   constexpr int NS = C::NS;
   extern __shared__ uint8_t dsm_raw[];
   uint8_t* dsm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = dsm;
-  uint8_t* ring = sQ + C::Q_BYTES;
+  uint8_t* sQ = dsm;  // [NQ][Q_BYTES]: item i uses buffer i % NQ
+  uint8_t* ring = sQ + C::NQ * C::Q_BYTES;  // K slots [0, NK), then V slots
+  uint8_t* vring = ring + C::NK * C::KV_BYTES;
   float* sbuf = reinterpret_cast<float*>(ring + NS * C::KV_BYTES);
 
   __shared__ Bars bars;
@@ -229,21 +247,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = tid >> 5;
 
   if (tid == 0) {
-    for (int s = 0; s < NS; ++s) {
-      mbar_init(&bars.full[s], 1);
-      mbar_init(&bars.empty[s], 1);
+    for (int s = 0; s < C::NK; ++s) {
+      mbar_init(&bars.kfull[s], 1);
+      mbar_init(&bars.kempty[s], 1);
     }
-    mbar_init(&bars.q_full, 1);
-    mbar_init(&bars.q_free, 128);
+    for (int s = 0; s < C::NV; ++s) {
+      mbar_init(&bars.vfull[s], 1);
+      mbar_init(&bars.vempty[s], 1);
+    }
     for (int b = 0; b < 2; ++b) {
+      mbar_init(&bars.q_full[b], 1);
+      mbar_init(&bars.q_free[b], C::QTMEM ? 128 : 1);  // the epilogue's copy, or the last QK
       mbar_init(&bars.qt_ready[b], 128);
-      mbar_init(&bars.s_full[b], 1);
-      mbar_init(&bars.p_full[b], 128);
       mbar_init(&bars.l_ready[b], 128);
       mbar_init(&bars.l_free[b], 128);
     }
-    mbar_init(&bars.pv_done[0], 1);
-    mbar_init(&bars.pv_done[1], 1);
+    for (int b = 0; b < C::NSB; ++b) {
+      mbar_init(&bars.s_full[b], 1);
+      mbar_init(&bars.p_full[b], 128);
+      mbar_init(&bars.pv_done[b], 1);
+    }
     mbar_init(&bars.o_full, 1);
     mbar_init(&bars.o_free, 128);
     mbar_init(&bars.drain, 1);
@@ -275,19 +298,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       auto load_q = [&](long long item) {
         const Work wq = decode_work<MODE>(p, item);
-        if (nq >= 1 && !wait_bounded(&bars.q_free, (nq - 1) & 1, &abort_sh, p.err)) return false;
-        mbar_arrive_expect_tx(&bars.q_full, C::Q_BYTES);
+        // buffer qb held the Q of item nq - NQ: its last QK (or, Q in TMEM, the
+        // epilogue's copy) must have read it
+        const int qb = nq % C::NQ;
+        if (nq >= C::NQ && !wait_bounded(&bars.q_free[qb], ((nq / C::NQ) - 1) & 1, &abort_sh, p.err)) return false;
+        mbar_arrive_expect_tx(&bars.q_full[qb], C::Q_BYTES);
         for (int ch = 0; ch < C::CHUNKS; ++ch)
-          tma_load_3d(sQ + ch * (BM * 128), &tmQ, &bars.q_full, ch * 64, (int)wq.r0, wq.b * p.Hq + wq.h0);
+          tma_load_3d(sQ + qb * C::Q_BYTES + ch * (BM * 128), &tmQ, &bars.q_full[qb], ch * 64, (int)wq.r0,
+                      wq.b * p.Hq + wq.h0);
         ++nq;
         return true;
       };
-      auto load_kv = [&](const CUtensorMap* m, int row, int z) {
-        const int s = c % NS;
-        if (c >= NS && !wait_bounded(&bars.empty[s], ((c / NS) - 1) & 1, &abort_sh, p.err)) return false;
-        mbar_arrive_expect_tx(&bars.full[s], C::KV_BYTES);
+      // K tiles only: the V tiles have their own ring and producer (warp
+      // 11), so a K load never waits for a PV to free a slot.
+      auto load_k = [&](int row, int z) {
+        const int s = c % C::NK;
+        if (c >= C::NK && !wait_bounded(&bars.kempty[s], ((c / C::NK) - 1) & 1, &abort_sh, p.err)) return false;
+        mbar_arrive_expect_tx(&bars.kfull[s], C::KV_BYTES);
         for (int ch = 0; ch < C::CHUNKS; ++ch)
-          tma_load_3d(ring + s * C::KV_BYTES + ch * (BN * 128), m, &bars.full[s], ch * 64, row, z);
+          tma_load_3d(ring + s * C::KV_BYTES + ch * (BN * 128), &tmK, &bars.kfull[s], ch * 64, row, z);
         ++c;
         return true;
       };
@@ -324,52 +353,74 @@ __global__ void __launch_bounds__(kThreads, 1)
         long long nxt = -1;
         for (int j = 0; ok && j < w.T; ++j) {
           const int krow = (int)(tile_index(w, j) * BN);
-          ok = load_kv(&tmK, krow, kz) && load_kv(&tmV, krow, kz);
+          ok = load_k(krow, kz);
           if (ok && j == 0) {
             nxt = claim();
-            if (nxt >= 0) ok = load_q(nxt);
+            // with two Q buffers, or Q copied to TMEM, the next item's Q goes out at once
+            if ((C::NQ >= 2 || C::QTMEM) && nxt >= 0) ok = load_q(nxt);
           }
         }
+        // with one Q buffer it waits for this item's last QK, so it goes out
+        // after this item's K/V loads (which that QK needs)
+        if (C::NQ == 1 && !C::QTMEM && ok && nxt >= 0) ok = load_q(nxt);
         item = nxt;
       }
       if (DYN && !done) claim();  // the readers always see the end of the sequence
-      // Drain: only the last NS ring loads and the last Q load can be in flight.
-      for (int u = (c > NS ? c - NS : 0); u < c; ++u) wait_drain(&bars.full[u % NS], (u / NS) & 1, p.err);
-      if (nq > 0) wait_drain(&bars.q_full, (nq - 1) & 1, p.err);
+      // Drain: only the last NK K loads and the last Q loads can be in flight.
+      for (int u = (c > C::NK ? c - C::NK : 0); u < c; ++u) wait_drain(&bars.kfull[u % C::NK], (u / C::NK) & 1, p.err);
+      for (int k = (nq > C::NQ ? nq - C::NQ : 0); k < nq; ++k)
+        wait_drain(&bars.q_full[k % C::NQ], (k / C::NQ) & 1, p.err);
     }
   } else if (warp == 9) {
     // ================================================================ QK issuer
     regs_decrease<kRegsControl>();
     if ((tid & 31) == 0) {
-      // Shared-memory descriptor of ring slot 0; a slot or K-step adds its
-      // byte offset / 16 to the start-address field.
+      // Shared-memory descriptors of Q buffer 0 and ring slot 0; a buffer,
+      // slot or K-step adds its byte offset / 16 to the start-address field.
+      const uint64_t qdesc0 = sdesc_sw128(smem_u32(sQ), 16, 1024);
       const uint64_t kdesc0 = sdesc_sw128(smem_u32(ring), 16, 1024);
+      const bool rope = p.rope != nullptr;
       long long g = 0;
       bool ok = true;
       ItemReader<DYN, false> items{(long long)blockIdx.x};
       int i = 0;
       for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
         const Work w = decode_work<MODE>(p, item);
-        if (!wait_bounded(&bars.qt_ready[i & 1], (i >> 1) & 1, &abort_sh, p.err)) { ok = false; break; }
-        const uint32_t qt = tmem + C::COL_Q + (uint32_t)(i & 1) * 64;
+        // Q of item i: in TMEM buffer i & 1 (copied by the epilogue), or in smem
+        // buffer i % NQ (rotated in place first when RoPE is on)
+        const int qb = C::QTMEM ? (i & 1) : i % C::NQ;
+        uint64_t* qbar = (C::QTMEM || rope) ? &bars.qt_ready[qb] : &bars.q_full[qb];
+        if (!wait_bounded(qbar, (uint32_t)(C::QTMEM ? (i >> 1) : i / C::NQ) & 1, &abort_sh, p.err)) {
+          ok = false;
+          break;
+        }
+        const uint32_t qt = tmem + C::COL_Q + (uint32_t)qb * 64;
+        const uint64_t qd = qdesc0 + ((qb * C::Q_BYTES) >> 4);
         for (int j = 0; j < w.T; ++j, ++g) {
-          const int ks = (int)((2 * g) % NS);
-          const uint32_t kph = (uint32_t)((2 * g) / NS) & 1;
-          if (!wait_bounded(&bars.full[ks], kph, &abort_sh, p.err)) { ok = false; break; }
-          // S buffer g&1 held P(g-2): PV(g-2) must have read it.
-          if (g >= 2 && !wait_bounded(&bars.pv_done[g & 1], (uint32_t)((g - 2) >> 1) & 1, &abort_sh, p.err)) {
+          const int ks = (int)(g % C::NK);
+          const uint32_t kph = (uint32_t)(g / C::NK) & 1;
+          const int sbi = (int)(g % C::NSB);
+          if (!wait_bounded(&bars.kfull[ks], kph, &abort_sh, p.err)) { ok = false; break; }
+          // S buffer sbi held P(g-3): PV(g-3) must have read it.
+          if (g >= C::NSB &&
+              !wait_bounded(&bars.pv_done[sbi], (uint32_t)((g - C::NSB) / C::NSB) & 1, &abort_sh, p.err)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sb = tmem + C::COL_S + (uint32_t)(g & 1) * BN;
+          const uint32_t sb = tmem + C::COL_S + (uint32_t)sbi * BN;
           const uint64_t kd = kdesc0 + ((ks * C::KV_BYTES) >> 4);
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk)
-            mma_ts(sb, qt + kk * 8, kd + ((((kk >> 2) * (BN * 128)) + (kk & 3) * 32) >> 4), C::IDESC_QK,
-                   kk > 0 ? 1u : 0u);
-          mma_commit(&bars.s_full[g & 1]);
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t off = (((kk >> 2) * (BN * 128)) + (kk & 3) * 32) >> 4;
+            if (C::QTMEM)
+              mma_ts(sb, qt + kk * 8, kd + off, C::IDESC_QK, kk > 0 ? 1u : 0u);
+            else
+              mma_ss(sb, qd + off, kd + off, C::IDESC_QK, kk > 0 ? 1u : 0u);
+          }
+          mma_commit(&bars.s_full[sbi]);
         }
+        if (!C::QTMEM && ok) mma_commit(&bars.q_free[qb]);  // the item's last QK has read its Q
       }
       if (!ok)  // after an early exit, read the item queue to its end marker
         while (items.next(p, iq, &abort_sh) >= 0) {}
@@ -380,7 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ================================================================ PV issuer
     regs_decrease<kRegsControl>();
     if ((tid & 31) == 0) {
-      const uint64_t vdesc0 = sdesc_sw128(smem_u32(ring), BN * 128, 1024);
+      const uint64_t vdesc0 = sdesc_sw128(smem_u32(vring), BN * 128, 1024);
       long long g = 0;
       bool ok = true;
       ItemReader<DYN, false> items{(long long)blockIdx.x};
@@ -388,21 +439,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
         const Work w = decode_work<MODE>(p, item);
         for (int j = 0; j < w.T; ++j, ++g) {
-          const int vs = (int)((2 * g + 1) % NS);
-          const uint32_t vph = (uint32_t)((2 * g + 1) / NS) & 1;
-          if (!wait_bounded(&bars.p_full[g & 1], (g >> 1) & 1, &abort_sh, p.err)) { ok = false; break; }
-          if (!wait_bounded(&bars.full[vs], vph, &abort_sh, p.err)) { ok = false; break; }
+          const int vs = (int)(g % C::NV);
+          const uint32_t vph = (uint32_t)(g / C::NV) & 1;
+          const int sbi = (int)(g % C::NSB);
+          if (!wait_bounded(&bars.p_full[sbi], (uint32_t)(g / C::NSB) & 1, &abort_sh, p.err)) { ok = false; break; }
+          if (!wait_bounded(&bars.vfull[vs], vph, &abort_sh, p.err)) { ok = false; break; }
           // The epilogue must have read the previous item's O.
           if (j == 0 && i >= 1 && !wait_bounded(&bars.o_free, (i - 1) & 1, &abort_sh, p.err)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t sb = tmem + C::COL_S + (uint32_t)(g & 1) * BN;
+          const uint32_t sb = tmem + C::COL_S + (uint32_t)sbi * BN;
           const uint64_t vd = vdesc0 + ((vs * C::KV_BYTES) >> 4);
           mma_ts(tmem + C::COL_O, sb, vd, C::IDESC_PV, j == 0 ? 0u : 1u);
 #pragma unroll
           for (int kk = 1; kk < BN / 16; ++kk)
             mma_ts(tmem + C::COL_O, sb + kk * 8, vd + ((kk * 2048) >> 4), C::IDESC_PV, 1u);
-          mma_commit(&bars.pv_done[g & 1]);
-          mma_commit(&bars.empty[vs]);
+          mma_commit(&bars.pv_done[sbi]);
+          mma_commit(&bars.vempty[vs]);
           if (j == w.T - 1) mma_commit(&bars.o_full);
         }
       }
@@ -412,8 +464,32 @@ __global__ void __launch_bounds__(kThreads, 1)
       wait_drain(&bars.drain2, 0, p.err);
     }
   } else if (warp == 11) {
-    // idle warp of the control warpgroup
+    // ================================================================ V producer
     regs_decrease<kRegsControl>();
+    if ((tid & 31) == 0) {
+      int c = 0;
+      bool ok = true;
+      ItemReader<DYN, false> items{(long long)blockIdx.x};
+      for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh)) {
+        const Work w = decode_work<MODE>(p, item);
+        const int kz = w.b * p.Hkv + w.g;
+        for (int j = 0; ok && j < w.T; ++j) {
+          const int s = c % C::NV;
+          if (c >= C::NV && !wait_bounded(&bars.vempty[s], ((c / C::NV) - 1) & 1, &abort_sh, p.err)) {
+            ok = false;
+            break;
+          }
+          const int krow = (int)(tile_index(w, j) * BN);
+          mbar_arrive_expect_tx(&bars.vfull[s], C::KV_BYTES);
+          for (int ch = 0; ch < C::CHUNKS; ++ch)
+            tma_load_3d(vring + s * C::KV_BYTES + ch * (BN * 128), &tmV, &bars.vfull[s], ch * 64, krow, kz);
+          ++c;
+        }
+      }
+      if (!ok)  // after an early exit, read the item queue to its end marker
+        while (items.next(p, iq, &abort_sh) >= 0) {}
+      for (int u = (c > C::NV ? c - C::NV : 0); u < c; ++u) wait_drain(&bars.vfull[u % C::NV], (u / C::NV) & 1, p.err);
+    }
   } else if (warp < 4) {
     // ================================================================ softmax
     regs_increase<kRegsCompute>();
@@ -434,14 +510,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       unmasked_tiles<MODE>(p, w, j_plain0, j_plain1);
       float m_run = -INFINITY, l_run = 0.f;
       for (int j = 0; ok && j < w.T; ++j, ++g) {
-        if (!__all_sync(kFull, wait_bounded(&bars.s_full[g & 1], (g >> 1) & 1, &abort_sh, p.err))) {
+        const int sbi = (int)(g % C::NSB);
+        if (!__all_sync(kFull, wait_bounded(&bars.s_full[sbi], (uint32_t)(g / C::NSB) & 1, &abort_sh, p.err))) {
           ok = false;
           break;
         }
-        // S(g) landed, so QK(g) has read its K tile (ring position 2g).
-        if (t == 0) mbar_arrive(&bars.empty[(2 * g) % NS]);
+        // S(g) landed, so QK(g) has read its K tile.
+        if (t == 0) mbar_arrive(&bars.kempty[g % C::NK]);
         tc_fence_after();
-        const uint32_t sb = C::COL_S + (uint32_t)(g & 1) * BN;
+        const uint32_t sb = C::COL_S + (uint32_t)sbi * BN;
         float s[BN];
         tmem_ld_row<BN>(tmem + la + sb, s);
         if (j < j_plain0 || j >= j_plain1) {
@@ -500,11 +577,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         f2_unpack(acc[2], a4, a5);
         f2_unpack(acc[3], a6, a7);
         const float l_tile = ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
-        // Rescale O (rare): PV(g-1) must have landed.  QK(g) waited for PV(g-2),
-        // and PV(g+1) needs this thread's P(g+1), so the parity of PV(g-1) on
-        // its buffer is unambiguous.
+        // Rescale O (rare): PV(g-1) must have landed.  QK(g-1) waited for
+        // PV(g-4), and PV(g+2) needs this thread's P(g+2), so the parity of
+        // PV(g-1) on its buffer is unambiguous.
         if (__any_sync(kFull, rescale)) {
-          if (!__all_sync(kFull, wait_bounded(&bars.pv_done[(g - 1) & 1], (uint32_t)((g - 1) >> 1) & 1, &abort_sh, p.err))) {
+          const int pb = (int)((g - 1) % C::NSB);
+          if (!__all_sync(kFull, wait_bounded(&bars.pv_done[pb], (uint32_t)((g - 1) / C::NSB) & 1, &abort_sh, p.err))) {
             ok = false;
             break;
           }
@@ -532,7 +610,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tmem_st_wait();
         tc_fence_before();
-        mbar_arrive(&bars.p_full[g & 1]);
+        mbar_arrive(&bars.p_full[sbi]);
       }
       if (!ok) continue;  // keep reading the item sequence to its end
       // Publish this item's row sum and max to the epilogue.
@@ -553,8 +631,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     int nq = 0;
     // Q of an item: swizzled smem rows -> TMEM lanes (bf16 pairs), the A
     // operand of S = Q K^T.
+    // RoPE (Sec. 2), rotate-half, when Q comes unrotated: each row of the
+    // item's Q tile turns in place in its smem buffer before its first QK.
+    // Channel c turns with channel c + D/2 by the angle of the row's position;
+    // word k of r holds channels 2k and 2k + 1, its partner word is k + D/4.
+    // fp32, one rounding to bf16.  Without RoPE the QK reads the TMA'd tile.
+    // Q in TMEM: the item's Q tile, swizzled smem rows -> TMEM lanes (bf16
+    // pairs), rotated on the way when RoPE is on; frees the smem buffer.
     auto copy_q = [&](int buf, long long qitem) {
-      ok = ok && __all_sync(kFull, wait_sleepy(&bars.q_full, nq & 1, &abort_sh, p.err));
+      ok = ok && __all_sync(kFull, wait_sleepy(&bars.q_full[0], nq & 1, &abort_sh, p.err));
       ++nq;
       if (ok) {
         uint32_t r[D / 2];
@@ -570,9 +655,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             r[ch * 32 + pc * 4 + 3] = v.w;
           }
         if (p.rope != nullptr) {
-          // RoPE (Sec. 2), rotate-half: channel c turns with channel c + D/2 by
-          // the angle of the row's position; word k of r holds channels 2k and
-          // 2k + 1, its partner word is k + D/4.  fp32, one rounding to bf16.
           const Work wq = decode_work<MODE>(p, qitem);
           long long qrow, qsample;
           int qhead;
@@ -601,15 +683,60 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_proxy_async_smem();  // the next TMA write of sQ follows these reads
       tc_fence_before();
       mbar_arrive(&bars.qt_ready[buf]);
-      mbar_arrive(&bars.q_free);
+      mbar_arrive(&bars.q_free[0]);
+    };
+    auto rotate_q = [&](int buf, long long qitem) {
+      if (C::QTMEM) {
+        copy_q(buf, qitem);
+        return;
+      }
+      if (p.rope == nullptr) return;
+      ok = ok && __all_sync(kFull, wait_sleepy(&bars.q_full[buf], (nq / C::NQ) & 1, &abort_sh, p.err));
+      ++nq;
+      const Work wq = decode_work<MODE>(p, qitem);
+      long long qrow, qsample;
+      int qhead;
+      if (ok && lane_row<MODE>(p, wq, e, qrow, qsample, qhead)) {
+        uint8_t* q = sQ + buf * C::Q_BYTES;
+        uint32_t r[D / 2];
+#pragma unroll
+        for (int ch = 0; ch < C::CHUNKS; ++ch)
+#pragma unroll
+          for (int pc = 0; pc < 8; ++pc) {
+            const uint4 v = *reinterpret_cast<const uint4*>(q + ch * (BM * 128) + e * 128 + ((pc ^ (e & 7)) * 16));
+            r[ch * 32 + pc * 4 + 0] = v.x;
+            r[ch * 32 + pc * 4 + 1] = v.y;
+            r[ch * 32 + pc * 4 + 2] = v.z;
+            r[ch * 32 + pc * 4 + 3] = v.w;
+          }
+        const float4* cs = reinterpret_cast<const float4*>(p.rope + qrow * D);
+#pragma unroll
+        for (int k = 0; k < D / 4; ++k) {
+          const float4 t = __ldg(cs + k);  // (cos, sin) of channels 2k, 2k + 1
+          const float a0 = __uint_as_float(r[k] << 16), a1 = __uint_as_float(r[k] & 0xffff0000u);
+          const float b0 = __uint_as_float(r[k + D / 4] << 16);
+          const float b1 = __uint_as_float(r[k + D / 4] & 0xffff0000u);
+          r[k] = pack_bf16x2(a0 * t.x - b0 * t.y, a1 * t.z - b1 * t.w);
+          r[k + D / 4] = pack_bf16x2(b0 * t.x + a0 * t.y, b1 * t.z + a1 * t.w);
+        }
+#pragma unroll
+        for (int ch = 0; ch < C::CHUNKS; ++ch)
+#pragma unroll
+          for (int pc = 0; pc < 8; ++pc)
+            *reinterpret_cast<uint4*>(q + ch * (BM * 128) + e * 128 + ((pc ^ (e & 7)) * 16)) =
+                make_uint4(r[ch * 32 + pc * 4 + 0], r[ch * 32 + pc * 4 + 1], r[ch * 32 + pc * 4 + 2],
+                           r[ch * 32 + pc * 4 + 3]);
+      }
+      fence_proxy_async_smem();  // the tensor core reads the rotated tile
+      mbar_arrive(&bars.qt_ready[buf]);
     };
     ItemReader<DYN, true> items{(long long)blockIdx.x};
     long long item = items.next(p, iq, &abort_sh);
-    if (item >= 0) copy_q(0, item);
+    if (item >= 0) rotate_q(0, item);
     for (int i = 0; item >= 0; ++i) {
       const Work w = decode_work<MODE>(p, item);
       const long long nxt = items.next(p, iq, &abort_sh);
-      if (nxt >= 0) copy_q((i + 1) & 1, nxt);
+      if (nxt >= 0) rotate_q(C::QTMEM ? ((i + 1) & 1) : (i + 1) % C::NQ, nxt);
       long long row, sample;
       int head;
       const bool row_ok = lane_row<MODE>(p, w, e, row, sample, head);

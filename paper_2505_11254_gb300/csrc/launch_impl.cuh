@@ -11,7 +11,7 @@ template <int D, int MODE, int EPI>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
                         long long n_items, cudaStream_t s) {
   auto kfn = attn_kernel<D, MODE, EPI>;
-  cudaError_t e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<D>::SMEM);
+  cudaError_t e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<D, MODE>::SMEM);
   if (e != cudaSuccess) return e;
   if (n_items <= 0) return cudaSuccess;
   int dev = 0, sms = 0;
@@ -20,7 +20,7 @@ cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUte
   Params q = p;
   q.n_items = n_items;
   const long long grid = n_items < sms ? n_items : sms;
-  kfn<<<(unsigned)grid, kThreads, Cfg<D>::SMEM, s>>>(tq, tk, tv, q);
+  kfn<<<(unsigned)grid, kThreads, Cfg<D, MODE>::SMEM, s>>>(tq, tk, tv, q);
   return cudaGetLastError();
 }
 

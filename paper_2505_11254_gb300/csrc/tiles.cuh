@@ -155,12 +155,27 @@ __host__ __device__ inline Work decode_strided_dense(const Params& p, long long 
 // batch) so the G query heads that share K/V run side by side.
 __host__ __device__ inline Work decode_sparse(const Params& p, long long lin) {
   Work w;
-  int hl = (int)(lin % p.G);
-  lin /= p.G;
-  long long qt = lin % p.qtiles;
-  lin /= p.qtiles;
-  w.g = (int)(lin % p.Hkv);
-  w.b = (int)(lin / p.Hkv);
+  int hl;
+  long long qt;
+  if (lin >= 0 && lin <= 0xffffffffLL && p.qtiles <= 0xffffffffLL) {
+    // 32-bit divisions (a 64-bit division by a runtime value is a long
+    // software sequence on the item-start path of every role); the same
+    // quotients
+    uint32_t l = (uint32_t)lin;
+    hl = (int)(l % (uint32_t)p.G);
+    l /= (uint32_t)p.G;
+    qt = l % (uint32_t)p.qtiles;
+    l /= (uint32_t)p.qtiles;
+    w.g = (int)(l % (uint32_t)p.Hkv);
+    w.b = (int)(l / (uint32_t)p.Hkv);
+  } else {
+    hl = (int)(lin % p.G);
+    lin /= p.G;
+    qt = lin % p.qtiles;
+    lin /= p.qtiles;
+    w.g = (int)(lin % p.Hkv);
+    w.b = (int)(lin / p.Hkv);
+  }
   w.h0 = w.g * p.G + hl;
   w.r0 = qt * BM;
   w.r_last = lmin(w.r0 + BM, p.N) - 1;
