@@ -523,21 +523,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld_row<BN>(tmem + la + sb, s);
         if (j < j_plain0 || j >= j_plain1) {
           // Visible key offsets c of this tile: lo <= c <= hi (window and
-          // causality), plus c < se (sinks).  Branch-free selects; the sink
-          // term only in tiles that hold sink keys.
+          // causality), plus c < se (sinks).  Per 32-key chunk the warp votes:
+          // a chunk no row of the warp sees becomes -inf by plain moves, a chunk
+          // every row sees whole is left alone, and only the mixed chunks (on
+          // the diagonal tile one per warp) take the per-key test.
           const long long k0 = tile_index(w, j) * BN;
           const int hi = (int)lmax(-1, lmin(BN - 1, row - k0));
           int lo = (MODE == MODE_STRIDED_DENSE) ? 0 : (int)lmax(0, lmin(BN, row - p.window + 1 - k0));
           if (hi < lo) lo = BN + 1;  // empty range: (uint)(c - lo) is then above any width
           const uint32_t width = hi >= lo ? (uint32_t)(hi - lo) : 0u;
-          if (MODE != MODE_STRIDED_DENSE && k0 < p.n_sink) {
-            const int se = (int)lmin(lmin(BN, (long long)p.n_sink - k0), (long long)hi + 1);
+          const int se = (MODE != MODE_STRIDED_DENSE && k0 < p.n_sink)
+                             ? (int)lmin(lmin(BN, (long long)p.n_sink - k0), (long long)hi + 1)
+                             : 0;
 #pragma unroll
-            for (int c = 0; c < BN; ++c)
-              s[c] = ((uint32_t)(c - lo) <= width || c < se) ? s[c] : -INFINITY;
-          } else {
+          for (int q = 0; q < BN / 32; ++q) {
+            const int c0 = 32 * q, c1 = c0 + 31;
+            const bool all = (lo <= c0 && c1 <= hi) || c1 < se;
+            if (!__all_sync(kFull, all)) {
 #pragma unroll
-            for (int c = 0; c < BN; ++c) s[c] = ((uint32_t)(c - lo) <= width) ? s[c] : -INFINITY;
+              for (int c = c0; c <= c1; ++c) s[c] = ((uint32_t)(c - lo) <= width || c < se) ? s[c] : -INFINITY;
+            }
           }
         }
         float mx[4];
