@@ -138,3 +138,28 @@ def test_timeout_path_reports_and_recovers():
     out = binding.delta_attn_prefill(q, k, v, 4, 32, 16)
     assert binding.check() == binding.DA_OK
     assert_close(out, ref["A"], "after timeout")
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_score_jump_inside_one_key_tile(d):
+    """Keys 64..127 and 320..383 scaled x32 give score jumps of more than
+    64 log2 units: inside the first key tile of rows 64..127, and, for the
+    rows past 384, in a tile that comes after others, so the lazy rescale of
+    O and the row sum (taken only past that threshold) runs in the middle of
+    rows, in both the sink+window and the dense kernels.
+    Such sharp rows return nearly single values of v, and A = S + D - S_k can
+    reach twice their range, so v is scaled by 1/8 (exact in bf16) to keep
+    the bf16 rounding of the output itself well inside the tolerance."""
+    B, Hq, Hkv, N, s, w, gamma = 1, 2, 1, 700, 4, 200, 16
+    q, k, v = rand_qkv(B, Hq, Hkv, N, d, seed=11 + d)
+    k, v = k.clone(), v * 0.125
+    k[:, :, 64:128] *= 32
+    k[:, :, 320:384] *= 32
+    ref = oracle_full(q, k, v, s, w, gamma)
+    out = binding.delta_attn_prefill(q, k, v, s, w, gamma)
+    o_sp = binding.sparse_window_attn(q, k, v, s, w, gamma)
+    d_samp = binding.strided_dense_attn(q, k, v, gamma)
+    assert binding.check() == binding.DA_OK
+    assert_close(out, ref["A"], "prefill")
+    assert_close(o_sp, ref["S"], "sparse_window_attn")
+    assert_close(d_samp, ref["D"], "strided_dense_attn")
