@@ -24,7 +24,7 @@
 //              wait for a PV to free a slot.
 // Registers: launched at 168 per thread (384 x 168 = 64512); the third
 // warpgroup gives back to 72 and the softmax and epilogue warpgroups grow to
-// 232 + 200 (light epilogues) or 216 + 216, so 128 x (432 + 72) = 64512 exactly.
+// 216, so 2 x 128 x 216 + 128 x 72 = 64512 exactly.
 // TMEM (512 columns): S/P triple buffer [0,128) [128,256) [256,384), O
 // [384, 384 + D).  Three S buffers let QK run up to three tiles ahead of the
 // softmax, so the chain softmax(g) -> PV(g) -> QK(g+3) spans three tiles.
@@ -46,18 +46,9 @@
 namespace da {
 
 constexpr int kThreads = 384;
-constexpr int kRegsControl = 72;  // producer / MMA warpgroup
-// Softmax and epilogue warpgroups: the softmax takes 16 more registers where
-// the epilogue is light (sparse rows plus at most a precomputed Delta); the
-// split-K merge and the smoothed-Delta epilogues keep an even split.
-template <int EPI>
-struct Regs {
-  static constexpr bool heavy_epi = (EPI == EPI_DENSE_F32 || EPI == EPI_DENSE_BF16 || EPI == EPI_FUSED_SMOOTH);
-  static constexpr int softmax = heavy_epi ? 216 : 232;
-  static constexpr int epilogue = heavy_epi ? 216 : 200;
-  static_assert(128 * (softmax + epilogue + kRegsControl) <= kThreads * 168, "register split above the launch total");
-  static_assert(softmax % 8 == 0 && epilogue % 8 == 0, "setmaxnreg takes multiples of 8");
-};
+constexpr int kRegsCompute = 216;  // softmax and epilogue warpgroups
+constexpr int kRegsControl = 72;   // producer / MMA warpgroup
+static_assert(2 * 128 * kRegsCompute + 128 * kRegsControl <= kThreads * 168, "register split above the launch total");
 // O and the row sum are rescaled only when the running max grows by more than
 // this many log2 units.  Until then P = 2^(s - m) can reach 2^64: bf16 and fp32
 // share the 8-bit exponent, and 2^64 x 2^20 keys x |v| stays far below the
@@ -501,7 +492,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp < 4) {
     // ================================================================ softmax
-    regs_increase<Regs<EPI>::softmax>();
+    regs_increase<kRegsCompute>();
     const int t = tid;
     const uint32_t la = lane_base(warp);
     const float scale = p.scale_log2;
@@ -533,10 +524,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (j < j_plain0 || j >= j_plain1) {
           // Visible key offsets c of this tile: lo <= c <= hi (window and
           // causality), plus c < se (sinks).  Per 32-key chunk the warp votes:
-          // a chunk every row sees whole is left alone, a chunk no row of the
-          // warp sees becomes -inf (a min with -inf held in a register: written
-          // as a constant store, the compiler spills), and only the mixed
-          // chunks (on the diagonal tile one per warp) take the per-key test.
+          // a chunk every row of the warp sees whole is left alone; every other
+          // chunk takes the per-key test (a second vote that set fully hidden
+          // chunks to -inf directly cost 7 % at window 512).
           const long long k0 = tile_index(w, j) * BN;
           const int hi = (int)lmax(-1, lmin(BN - 1, row - k0));
           int lo = (MODE == MODE_STRIDED_DENSE) ? 0 : (int)lmax(0, lmin(BN, row - p.window + 1 - k0));
@@ -549,17 +539,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int q = 0; q < BN / 32; ++q) {
             const int c0 = 32 * q, c1 = c0 + 31;
             const bool all = (lo <= c0 && c1 <= hi) || c1 < se;
-            const bool none = (c1 < lo || c0 > hi) && c0 >= se;
             if (!__all_sync(kFull, all)) {
-              if (__all_sync(kFull, none)) {
-                float ninf;
-                asm("mov.b32 %0, 0xff800000;" : "=f"(ninf));
 #pragma unroll
-                for (int c = c0; c <= c1; ++c) s[c] = fminf(s[c], ninf);
-              } else {
-#pragma unroll
-                for (int c = c0; c <= c1; ++c) s[c] = ((uint32_t)(c - lo) <= width || c < se) ? s[c] : -INFINITY;
-              }
+              for (int c = c0; c <= c1; ++c) s[c] = ((uint32_t)(c - lo) <= width || c < se) ? s[c] : -INFINITY;
             }
           }
         }
@@ -647,7 +629,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ================================================================ epilogue
-    regs_increase<Regs<EPI>::epilogue>();
+    regs_increase<kRegsCompute>();
     const int e = tid - 128;  // TMEM lane = query row of the tile
     const uint32_t la = lane_base(warp);
     bool ok = true;
