@@ -14,9 +14,11 @@
 //              RoPE is on, then reads O out of TMEM, releases it, normalises,
 //              applies the Delta correction and writes the output.
 //   warp 8     TMA producer: Q of the next item, K tiles through their ring.
-//   warp 9     QK issuer: S = Q K^T (Q and K from smem) once its K tile has
-//              landed and PV(g-3) has freed the S buffer; Q is double-buffered
-//              in smem (item i in buffer i & 1).
+//   warp 9     QK issuer: S = Q K^T once its K tile has landed and the PV
+//              that last read the S buffer has completed.  Sink + window
+//              passes: Q from smem (one buffer at d = 128, reloaded after the
+//              item's last QK; two at d = 64).  Dense pass: Q from TMEM
+//              (two buffers, filled by the epilogue warps).
 //   warp 10    PV issuer: O += P V (P from TMEM, V from smem) once the softmax
 //              has written P(g).  Two issuing threads keep the tensor pipe fed:
 //              neither waits on the other's inputs.
@@ -25,9 +27,10 @@
 // Registers: launched at 168 per thread (384 x 168 = 64512); the third
 // warpgroup gives back to 72 and the softmax and epilogue warpgroups grow to
 // 216, so 2 x 128 x 216 + 128 x 72 = 64512 exactly.
-// TMEM (512 columns): S/P triple buffer [0,128) [128,256) [256,384), O
-// [384, 384 + D).  Three S buffers let QK run up to three tiles ahead of the
-// softmax, so the chain softmax(g) -> PV(g) -> QK(g+3) spans three tiles.
+// TMEM (512 columns), two layouts (see Cfg): sink + window passes hold an
+// S/P triple buffer and O, so QK may run three tiles ahead of the softmax and
+// the chain softmax(g) -> PV(g) -> QK(g+3) spans three tiles; the dense pass
+// holds Q (two buffers), an S/P double buffer and O.
 // Every wait is bounded: past its limit a wait sets the CTA's abort flag and
 // the device status word, the roles stop working (keeping every named barrier
 // and warp-collective instruction uniform), drain their in-flight copies and
@@ -401,7 +404,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t kph = (uint32_t)(g / C::NK) & 1;
           const int sbi = (int)(g % C::NSB);
           if (!wait_bounded(&bars.kfull[ks], kph, &abort_sh, p.err)) { ok = false; break; }
-          // S buffer sbi held P(g-3): PV(g-3) must have read it.
+          // S buffer sbi held P(g - NSB): that PV must have read it.
           if (g >= C::NSB &&
               !wait_bounded(&bars.pv_done[sbi], (uint32_t)((g - C::NSB) / C::NSB) & 1, &abort_sh, p.err)) {
             ok = false;
@@ -583,8 +586,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         f2_unpack(acc[3], a6, a7);
         const float l_tile = ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
         // Rescale O (rare): PV(g-1) must have landed.  QK(g-1) waited for
-        // PV(g-4), and PV(g+2) needs this thread's P(g+2), so the parity of
-        // PV(g-1) on its buffer is unambiguous.
+        // PV(g-1-NSB), and the next PV on that buffer needs this thread's
+        // P(g-1+NSB), so the parity of PV(g-1) on its buffer is unambiguous.
         if (__any_sync(kFull, rescale)) {
           const int pb = (int)((g - 1) % C::NSB);
           if (!__all_sync(kFull, wait_bounded(&bars.pv_done[pb], (uint32_t)((g - 1) / C::NSB) & 1, &abort_sh, p.err))) {
