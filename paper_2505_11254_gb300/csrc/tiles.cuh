@@ -158,9 +158,9 @@ __host__ __device__ inline Work decode_sparse(const Params& p, long long lin) {
   int hl;
   long long qt;
   if (lin >= 0 && lin <= 0xffffffffLL && p.qtiles <= 0xffffffffLL) {
-    // 32-bit divisions (a 64-bit division by a runtime value is a long
-    // software sequence on the item-start path of every role); the same
-    // quotients
+    // 32-bit divisions when the values fit, with the same quotients as the
+    // 64-bit path below (a 64-bit division by a runtime value is a long
+    // software sequence on the item-start path of every role).
     uint32_t l = (uint32_t)lin;
     hl = (int)(l % (uint32_t)p.G);
     l /= (uint32_t)p.G;
