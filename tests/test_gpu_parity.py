@@ -32,6 +32,8 @@ CASES = [
     (1, 4, 1, 1536, 128, 4, 300, 48),     # gamma 48 (not a divisor of 128), split-K
     (1, 4, 2, 700, 128, 4, 100, 4),       # gamma 4 at d = 128: Delta built in a separate pass
     (2, 2, 2, 300, 128, 2, 40, 2),        # gamma 2
+    (1, 16, 1, 400, 128, 4, 64, 16),      # GQA 16: 16 heads x 8 samples per dense tile
+    (1, 6, 2, 350, 64, 3, 50, 8),         # GQA 3 (not a power of two): one head per dense tile
     (1, 4, 4, 520, 64, 4, 64, 4),         # gamma 4 at d = 64: fused in the tile
 ]
 
