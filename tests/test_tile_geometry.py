@@ -1,7 +1,9 @@
 """Host logic of the kernels' tile geometry (tiles.cuh, compiled as plain C++
 with g++): the per-item range of tiles that skip the element-wise mask agrees
-with the per-tile predicate, and no skipped tile holds an invisible
-(row, key) pair, over many shapes, all three modes and the dense tail."""
+with the per-tile predicate, no skipped tile holds an invisible (row, key)
+pair, the split-K units cover each dense M-tile once, and every lane maps to
+its query head's KV head with each (batch, head, row) held once, over many
+shapes, all three modes, the dense tail and the GQA head packings."""
 import os
 import shutil
 import subprocess

@@ -5,7 +5,9 @@
 // (row, key) pair of the tile is not visible (checked pair by pair against
 // the definition of the key sets), and the dense pass's split-K units cover
 // every M-tile's causal key range exactly once in the order the partial slots
-// and tickets assume.
+// and tickets assume.  For every head packing of the dense tiles (GQA 1, 2,
+// 3, 4 and 16), each lane's query head reads its own KV head (floor(h / G))
+// and every (batch, head, row or sample) sits in exactly one lane.
 #define __host__
 #define __device__
 #define __forceinline__ inline
@@ -26,10 +28,33 @@ static bool visible(const Params& p, int mode, long long row, long long key) {
 template <int MODE>
 static int check(const Params& p, long long items) {
   int bad = 0;
+  // every (b, query head, row or sample) is held by exactly one lane of one item
+  const long long per_head = MODE == MODE_SPARSE ? p.N : p.n_s;
+  std::vector<unsigned char> held(MODE == MODE_STRIDED_DENSE ? 0 : (size_t)p.B * p.Hq * per_head, 0);
   for (long long it = 0; it < items; ++it) {
     Work w = decode_work<MODE>(p, it);
     int j0, j1;
     unmasked_tiles<MODE>(p, w, j0, j1);
+    for (int t = 0; t < BM; ++t) {  // GQA: every lane's query head reads the item's KV head
+      long long row, sample;
+      int head;
+      if (!lane_row<MODE>(p, w, t, row, sample, head)) continue;
+      const bool head_ok = head >= 0 && head < p.Hq && head / p.G == w.g && w.b >= 0 && w.b < p.B;
+      if (!head_ok) {
+        if (bad < 5) std::printf("mode %d item %lld lane %d: head %d, kv head %d, G %d\n", MODE, it, t, head, w.g, p.G);
+        ++bad;
+        continue;
+      }
+      if (MODE != MODE_STRIDED_DENSE) {
+        const long long r = MODE == MODE_SPARSE ? row : sample;
+        unsigned char& h = held[((size_t)w.b * p.Hq + head) * per_head + r];
+        if (h) {
+          if (bad < 5) std::printf("mode %d: (b %d, head %d, %lld) held twice\n", MODE, w.b, head, r);
+          ++bad;
+        }
+        h = 1;
+      }
+    }
     for (int j = 0; j < w.T; ++j) {
       const bool need = tile_needs_mask<MODE>(p, w, j);
       const bool in_range = j >= j0 && j < j1;
@@ -55,6 +80,11 @@ static int check(const Params& p, long long items) {
       }
     }
   }
+  for (size_t i = 0; i < held.size(); ++i)
+    if (!held[i]) {
+      if (bad < 5) std::printf("mode %d: (b, head, row) %zu held by no lane\n", MODE, i);
+      ++bad;
+    }
   return bad;
 }
 
@@ -94,6 +124,52 @@ static int check_dense_units(const Params& p) {
   return bad;
 }
 
+// Hp query heads of one KV group share a dense tile when G is a power of two
+// up to 16 (R = 128 / Hp samples each); otherwise one head per tile.
+static void set_packing(Params& p) {
+  p.Hp = (p.G >= 2 && p.G <= 16 && (p.G & (p.G - 1)) == 0) ? p.G : 1;
+  p.R = BM / p.Hp;
+  p.groups_per_b = p.Hq / p.Hp;
+}
+
+static long long count_units(Params& p) {
+  p.mtiles = (p.n_s + p.R - 1) / p.R;
+  long long units = 0, multi = 0;
+  for (long long t = 0; t < p.mtiles; ++t) {
+    const long long nc = (strided_dense_len(p, t) + p.chunk - 1) / p.chunk;
+    units += nc;
+    if (nc > 1) multi += nc;
+  }
+  p.n_units = units * p.B * p.groups_per_b;
+  p.n_multi = multi * p.B * p.groups_per_b;
+  return p.n_units;
+}
+
+static int check_shape(int B, int Hq, int Hkv, long long N, long long win, int ns, int gm) {
+  int bad = 0;
+  Params p = {};
+  p.B = B; p.Hq = Hq; p.Hkv = Hkv; p.G = Hq / Hkv; p.N = N; p.n_sink = ns; p.window = win; p.gamma = gm;
+  p.n_s = (N + gm - 1) / gm;
+  set_packing(p);
+  p.qtiles = (N + BM - 1) / BM;
+  p.chunk = 3;
+  count_units(p);
+  bad += check<MODE_SPARSE>(p, (long long)p.B * p.Hq * p.qtiles);
+  bad += check<MODE_STRIDED_SPARSE>(p, (long long)p.B * p.groups_per_b * p.mtiles);
+  bad += check<MODE_STRIDED_DENSE>(p, p.n_units);
+  bad += check_dense_units(p);
+  // the dense tail: gamma 1 from row N - tail
+  for (long long tail : {1LL, 77LL, N}) {
+    if (tail > N) continue;
+    Params q = p;
+    q.gamma = 1; q.n_s = tail; q.row0 = N - tail;
+    count_units(q);
+    bad += check<MODE_STRIDED_DENSE>(q, q.n_units);
+    bad += check_dense_units(q);
+  }
+  return bad;
+}
+
 int main() {
   int bad = 0, cases = 0;
   const long long Ns[] = {1, 100, 128, 129, 1000, 4097, 20000};
@@ -104,46 +180,19 @@ int main() {
     for (long long win : windows)
       for (int ns : sinks)
         for (int gm : gammas) {
-          Params p = {};
-          p.B = 1; p.Hq = 4; p.Hkv = 2; p.G = 2; p.N = N; p.n_sink = ns; p.window = win; p.gamma = gm;
-          p.n_s = (N + gm - 1) / gm;
-          p.Hp = 2; p.R = BM / 2; p.groups_per_b = 2;
-          p.mtiles = (p.n_s + p.R - 1) / p.R;
-          p.qtiles = (N + BM - 1) / BM;
-          p.chunk = 3;
-          long long units = 0;
-          for (long long t = 0; t < p.mtiles; ++t) units += (strided_dense_len(p, t) + p.chunk - 1) / p.chunk;
-          p.n_units = units * p.B * p.groups_per_b;
-          bad += check<MODE_SPARSE>(p, (long long)p.B * p.Hq * p.qtiles);
-          bad += check<MODE_STRIDED_SPARSE>(p, (long long)p.B * p.groups_per_b * p.mtiles);
-          p.n_multi = 0;
-          for (long long t = 0; t < p.mtiles; ++t) {
-            const long long nc = (strided_dense_len(p, t) + p.chunk - 1) / p.chunk;
-            if (nc > 1) p.n_multi += nc;
-          }
-          p.n_multi *= (long long)p.B * p.groups_per_b;
-          bad += check<MODE_STRIDED_DENSE>(p, p.n_units);
-          bad += check_dense_units(p);
-          // the dense tail: gamma 1 from row N - tail
-          for (long long tail : {1LL, 77LL, N}) {
-            if (tail > N) continue;
-            Params q = p;
-            q.gamma = 1; q.n_s = tail; q.row0 = N - tail;
-            q.mtiles = (q.n_s + q.R - 1) / q.R;
-            long long u = 0;
-            for (long long t = 0; t < q.mtiles; ++t) u += (strided_dense_len(q, t) + q.chunk - 1) / q.chunk;
-            q.n_units = u * q.B * q.groups_per_b;
-            q.n_multi = 0;
-            for (long long t = 0; t < q.mtiles; ++t) {
-              const long long nc = (strided_dense_len(q, t) + q.chunk - 1) / q.chunk;
-              if (nc > 1) q.n_multi += nc;
-            }
-            q.n_multi *= (long long)q.B * q.groups_per_b;
-            bad += check<MODE_STRIDED_DENSE>(q, q.n_units);
-            bad += check_dense_units(q);
-          }
+          bad += check_shape(1, 4, 2, N, win, ns, gm);
           ++cases;
         }
+  // other head packings (GQA 1, 3, 4 with B = 2, 16) on a smaller grid
+  const int packs[][3] = {{1, 2, 2}, {1, 6, 2}, {2, 8, 2}, {1, 16, 1}};
+  for (const auto& hk : packs)
+    for (long long N : {1LL, 129LL, 1000LL, 4097LL})
+      for (long long win : {1LL, 64LL, 300LL, 2048LL})
+        for (int ns : {0, 4, 300})
+          for (int gm : {1, 3, 16, 64}) {
+            bad += check_shape(hk[0], hk[1], hk[2], N, win, ns, gm);
+            ++cases;
+          }
   std::printf("%d shapes, %d mismatches\n", cases, bad);
   return bad == 0 ? 0 : 1;
 }
