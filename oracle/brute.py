@@ -55,6 +55,28 @@ def smooth(kind, params, delta, N, gamma):
     return np.repeat(out, gamma, axis=0)[:N]
 
 
+def lemma1_terms(Qf, Kf, Vf, n_sink, window, gamma, b, h, k):
+    """Both sides of Lemma 1 for the sampled row i = k gamma of (b, h), from
+    the explicit score row: a = causal softmax, a* = sparse softmax, the
+    omitted set C(i) minus W(i).  H/(H+T) is the total causal-softmax weight of
+    the omitted keys; returns (lhs[d], rhs[d], H/(H+T))."""
+    N, d = Qf.shape[2], Qf.shape[3]
+    G = Qf.shape[1] // Kf.shape[1]
+    i = k * gamma
+    Kh, Vh = Kf[b, h // G], Vf[b, h // G]
+    col = np.arange(N)
+    causal = col <= i
+    sparse = causal & ((col > i - window) | (col < n_sink))
+    omitted = causal & ~sparse
+    scores = (Kh @ Qf[b, h, i]) / np.sqrt(d)
+    a = _masked_softmax(scores[None, :], causal[None, :])[0]
+    a_star = _masked_softmax(scores[None, :], sparse[None, :])[0]
+    delta = a @ Vh - a_star @ Vh
+    head = np.where(omitted, a, 0.0) @ Vh
+    frac = a[omitted].sum()
+    return np.abs(delta - head), frac * np.abs(Vh[sparse]).max(axis=0), frac
+
+
 def delta_attn(Qf, Kf, Vf, n_sink, window, gamma, mode="delta", tail_dense=0, smooth_kind="none",
                smooth_params=()):
     """Qf [B,Hq,N,d], Kf/Vf [B,Hkv,N,d] float64.  Returns (A_hat, S, D_full).

@@ -500,7 +500,7 @@ int oracle_lemma1(const uint16_t *Q, const uint16_t *K, const uint16_t *V,
             dense[c] += a * v;
             sparse[c] += as * v;
             if (!in_w) head[c] += a * v;
-            if (in_w && fabs(v) > vmax[c]) vmax[c] = fabs(v);
+            if ((in_w || MUTANT(14)) && fabs(v) > vmax[c]) vmax[c] = fabs(v);
         }
     }
     for (int c = 0; c < d; ++c) {

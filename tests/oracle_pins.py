@@ -15,7 +15,9 @@ What pins what:
                                 window = 1 (S_i = v_i), constant V, and the
                                 sampled-row identity A^V_{k gamma} = ~AV_k.
   * GQA head mapping         -> explicit repetition of the KV heads.
-  * Lemma 1                  -> the appendix inequality on every sample.
+  * Lemma 1                  -> the appendix inequality on every sample,
+                                and both of its sides in closed form under
+                                uniform scores (Q = 0).
   * whole-matrix restatement -> the numpy brute force (oracle/brute.py).
   * Eq. 2 decoding           -> the dense causal row at the token's position
                                 and torch scaled_dot_product_attention.
@@ -210,6 +212,53 @@ def pin_lemma1(lib=None):
     assert nontrivial > 0
 
 
+def pin_lemma1_uniform(lib=None):
+    """Lemma 1's terms in closed form.  With Q = 0 every score is 0, so over
+    the causal set C(i) (i + 1 keys) and the sparse set W(i): H = |C \\ W|,
+    T = |W|, H/(H+T) = 1 - |W|/(i+1); Delta minus the omitted-key term is
+    mean_W(v) (|W|/(i+1) - 1), so lhs = H/(H+T) |mean_W(v)|, and
+    rhs = H/(H+T) max_W |v|.  V carries large values on keys outside W(i), so
+    a maximum taken over any other set than W(i) shows."""
+    B, Hq, Hkv, N, d = 1, 2, 1, 80, 8
+    n_sink, window, gamma = 2, 9, 8
+    Q = const_bits((B, Hq, N, d), 0.0)
+    K = rand_bits(24, (B, Hkv, N, d))
+    v = f64(rand_bits(25, (B, Hkv, N, d)))
+    v[0, 0, n_sink:N - window] *= 16.0   # keys omitted by every late row
+    V = torch.from_numpy(v.astype(np.float32)).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    vv = f64(V)[0, 0]
+    checked = 0
+    for h in range(Hq):
+        for k in range(N // gamma):
+            i = k * gamma
+            j = np.arange(i + 1)
+            w_set = (j < n_sink) | (j > i - window)
+            frac = 1.0 - w_set.sum() / (i + 1.0)
+            lhs, rhs, f = oracle.lemma1(Q, K, V, n_sink, window, gamma, 0, h, k, lib=lib)
+            assert abs(f - frac) <= TOL, (h, k, f, frac)
+            assert np.abs(lhs - frac * np.abs(vv[j[w_set]].mean(axis=0))).max() <= TOL, (h, k)
+            assert np.abs(rhs - frac * np.abs(vv[j[w_set]]).max(axis=0)).max() <= TOL, (h, k)
+            checked += frac > 0
+    assert checked > 0
+
+
+def pin_lemma1_brute(lib=None):
+    """Lemma 1's terms equal the whole-matrix restatement (oracle/brute.py)
+    on random inputs with scaled sinks."""
+    B, Hq, Hkv, N, d = 2, 4, 2, 70, 16
+    Q, K, V = rand_bits(26, (B, Hq, N, d), 1.5), rand_bits(27, (B, Hkv, N, d), 1.5), rand_bits(28, (B, Hkv, N, d))
+    K[:, :, :3] = rand_bits(29, (B, Hkv, 3, d), 8.0)
+    Qf, Kf, Vf = f64(Q), f64(K), f64(V)
+    for (n_sink, window, gamma) in ((3, 10, 7), (0, 1, 5), (4, 64, 16)):
+        for b in range(B):
+            for h in range(Hq):
+                for k in range((N + gamma - 1) // gamma):
+                    lhs, rhs, f = oracle.lemma1(Q, K, V, n_sink, window, gamma, b, h, k, lib=lib)
+                    bl, br, bf = brute.lemma1_terms(Qf, Kf, Vf, n_sink, window, gamma, b, h, k)
+                    assert abs(f - bf) <= TOL and np.abs(lhs - bl).max() <= TOL and np.abs(rhs - br).max() <= TOL, \
+                        (n_sink, window, gamma, b, h, k)
+
+
 def pin_brute_force(lib=None):
     """The direct per-row evaluation equals the whole-matrix restatement of
     Alg. 1 (numpy) on small problems, over a sweep of gamma, window, sinks,
@@ -400,8 +449,8 @@ def pin_rope(lib=None):
 
 ALL_PINS = [pin_gamma1_is_sdpa, pin_full_window_is_sdpa, pin_zero_keys_closed_form,
             pin_window1_no_sink, pin_constant_values, pin_mask_structure,
-            pin_sampled_rows_are_dense, pin_gqa_repeat, pin_lemma1, pin_rows_agree,
+            pin_sampled_rows_are_dense, pin_gqa_repeat, pin_lemma1, pin_lemma1_uniform, pin_rows_agree,
             pin_smooth_reductions, pin_smooth_closed_forms, pin_decode, pin_rope]
 # The brute-force restatements are listed separately: the mutant test shows the
 # other pins catch every planted mistake without them.
-BRUTE_PINS = [pin_brute_force, pin_smooth_brute]
+BRUTE_PINS = [pin_brute_force, pin_smooth_brute, pin_lemma1_brute]

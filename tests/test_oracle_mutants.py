@@ -7,7 +7,9 @@ over the sparse set, Delta taken against the current row instead of the
 sample, a transposed K operand, and three smoothing slips (EMA weights
 swapped, the filter's velocity gain replaced by its position gain, the
 interpolation weight one row ahead), and a decode that leaves out the new
-token's own key, and a RoPE rotation in the wrong direction.  All of this runs on the CPU.
+token's own key, a RoPE rotation in the wrong direction, and Lemma 1's
+bound taken with the largest |v_j| over every causal key instead of W(i).
+All of this runs on the CPU.
 """
 import os
 import tempfile
@@ -31,6 +33,7 @@ MUTANTS = {
     11: "linear interpolation weight one row ahead",
     12: "decode without the new token's own key",
     13: "RoPE rotation in the wrong direction",
+    14: "Lemma 1 bound with the max |v| over every causal key",
 }
 
 _tmp = tempfile.mkdtemp(prefix="oracle_mutants_")
