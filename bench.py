@@ -19,9 +19,21 @@ dense kernel, then the sink+window kernel with the fused Delta epilogue.
                  (appendix "Implementation Details") and the three Delta
                  smoothing forms (appendix "Interpolation"), timed the same way
 
+  workloads      (default workload only) the million-token prefill with its
+                 dense baseline, and the B=4 sweep's window-512 gamma-64 point,
+                 through the same timed code
+
+The timed loop of --steps prefills is repeated back to back until the timed
+region lasts about one second (each repeat bracketed by a barrier and a
+device synchronize); ms_per_step is the mean over all timed steps, and the SM
+clocks are sampled every 20 ms inside that region.
+
 ``--impl reference`` times the oracle as the reference arm.  Multi-GPU: one
-process per GPU (torchrun), independent sequences per rank, no collective on
-the data path (weak scaling); barrier + max over ranks around the timed loop.
+process per GPU (torchrun), no collective on the data path; barrier + max over
+ranks around each timed loop.  ``--shard replicas`` (default) runs one
+independent sequence per rank (weak scaling); ``--shard heads`` splits one
+prefill by (batch, KV head) pairs (strong scaling), ``--gather`` then times an
+all-gather of O.
 """
 import argparse
 import hashlib
@@ -63,6 +75,12 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-variants", action="store_true", help="skip the Eq. 5 / dense-tail timings")
     ap.add_argument("--tail", type=int, default=1024, help="dense tail rows of the variant timings")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="skip the 1M-token and B=4 window-512 records of the default run")
+    ap.add_argument("--shard", choices=["replicas", "heads"], default="replicas",
+                    help="N GPUs: independent sequences (weak scaling) or one prefill split by (batch, KV head) "
+                         "pairs (strong scaling)")
+    ap.add_argument("--gather", action="store_true", help="with --shard heads: time an all-gather of O afterwards")
     return ap.parse_args()
 
 
@@ -125,10 +143,14 @@ def recorded_traffic(kernel, workload):
 
 # ------------------------------------------------------------------ clocks
 class ClockSampler:
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi sampled every 20 ms while the GPU works; only the samples
+    taken between mark_start() and mark_end() (host wall clock, which brackets
+    the timed loops) are kept."""
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
     REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+    PERIOD_MS = 20
 
     def __init__(self, local_index):
         vis = os.environ.get("CUDA_VISIBLE_DEVICES")
@@ -139,14 +161,29 @@ class ClockSampler:
                 idx = parts[local_index]
         self.idx = idx
         self.proc = None
+        self.t0 = self.t1 = None
 
     def start(self):
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits", "-i", self.idx,
-                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", str(self.PERIOD_MS)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
+
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
+
+    @staticmethod
+    def _when(stamp):
+        import datetime
+        try:
+            return datetime.datetime.strptime(stamp, "%Y/%m/%d %H:%M:%S.%f").timestamp()
+        except ValueError:
+            return None
 
     def stop(self):
         if self.proc is None:
@@ -157,22 +194,28 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
             out, _ = self.proc.communicate()
-        sm, smax, power, reasons = [], [], [], set()
+        sm, smax, power, reasons, outside = [], [], [], set(), 0
         for line in out.splitlines():
             f = [x.strip() for x in line.split(",")]
-            if len(f) < 9:
+            if len(f) < 10:
+                continue
+            when = self._when(f[0])
+            if when is not None and self.t0 is not None and not (self.t0 <= when <= (self.t1 or when)):
+                outside += 1
                 continue
             try:
-                sm.append(float(f[1]))
-                smax.append(float(f[2]))
-                power.append(float(f[3]))
+                sm.append(float(f[2]))
+                smax.append(float(f[3]))
+                power.append(float(f[4]))
             except ValueError:
                 continue
-            for name, val in zip(self.REASONS, f[5:9]):
+            for name, val in zip(self.REASONS, f[6:10]):
                 if val.lower().startswith("active"):
                     reasons.add(name)
         return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
-                "power_w_max": max(power) if power else None, "reasons": sorted(reasons), "samples": len(sm)}
+                "sm_mhz_min": min(sm) if sm else None, "power_w_max": max(power) if power else None,
+                "reasons": sorted(reasons), "samples": len(sm), "period_ms": self.PERIOD_MS,
+                "samples_outside_timed_region": outside}
 
 
 # ------------------------------------------------------------------ oracle legs
@@ -254,7 +297,7 @@ def run_reference(args, w, rep):
     }), flush=True)
 
 
-def config_of(w, n_gpus):
+def config_of(w, n_gpus, shard="replicas"):
     qkv = 2 * w.d * w.N * (w.B * w.Hq + 2 * w.B * w.Hkv)
     l2 = ("inputs larger than L2 (Q+K+V %.2f GiB vs 129 MB L2), no flush" % (qkv / 2 ** 30) if qkv > 129e6 else
           "inputs smaller than L2 (%.1f MB), no flush: not a headline configuration" % (qkv / 1e6))
@@ -262,7 +305,9 @@ def config_of(w, n_gpus):
             "window": w.window, "gamma": w.gamma, "rope_base": w.rope_base if w.rope else None,
             "sink_scale": w.sink_scale,
             "l2": l2,
-            "parallelism": "replicas: one independent sequence per GPU" if n_gpus > 1 else "single GPU"}
+            "parallelism": ("single GPU" if n_gpus == 1 else
+                            "head shards: one prefill, (batch, KV head) pairs split over %d GPUs" % n_gpus
+                            if shard == "heads" else "replicas: one independent sequence per GPU")}
 
 
 def time_variants(args, w, q, k, v, out, stream, restore):
@@ -383,18 +428,33 @@ def time_decode(w, q, k, v, stream):
             "note": "one token per sequence, all heads; split-K kernel + merge kernel (dependent launch) per call"}
 
 
-def run_ours(args, w, rep):
+KERNEL_NAMES = {1: ["dense_bf16"], 2: ["strided_dense_f32", "sink_window_fused_delta"],
+                3: ["strided_dense_f32", "strided_sparse_delta", "sink_window_delta"]}
+
+
+def kernel_flops(w, nk):
+    """Useful FLOPs of each kernel of the launch sequence (4d per unmasked
+    pair: the dense rows in the strided dense kernel, the sink+window rows in
+    the sink+window kernel; the strided sparse Delta pass adds none)."""
+    hq_flops = 4 * w.d * w.B * w.Hq
+    dense_f = hq_flops * flops.dense_pairs_per_head(w.N, w.gamma)
+    sparse_f = hq_flops * flops.sparse_pairs_per_head(w.N, w.n_sink, w.window)
+    return {1: [dense_f], 2: [dense_f, sparse_f], 3: [dense_f, 0, sparse_f]}[nk]
+
+
+def time_prefill(w, q, k, v, steps, warmup, rep, peaks, peak_src, local, min_seconds=1.0, max_repeats=25):
+    """Warm-up, then the timed loop of `steps` delta_attn_prefill calls,
+    repeated back to back (each repeat bracketed by a barrier and a device
+    synchronize, the max over ranks taken per repeat) until the timed region
+    lasts about `min_seconds` (about 50 clock samples at one per 20 ms).
+    The library records CUDA events between its
+    kernels on the launching stream, which give the per-kernel times.  Returns
+    (record, out) with out holding the last step's result."""
     from paper_2505_11254_gb300 import binding
-    world, rank, local = rep.world, rep.rank, rep.local
-    dev = torch.device("cuda", local)
-    torch.cuda.set_device(dev)
-    peaks, peak_src = load_peaks()
-    wr = w.with_(seed=rep.seed(w.seed))
-    q, k, v = generate(wr, device=dev)
-    info = binding.plan_info(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, w.gamma)
+    B, Hq, Hkv, N, d = q.shape[0], q.shape[1], k.shape[1], q.shape[2], q.shape[3]
+    info = binding.plan_info(B, Hq, Hkv, N, d, w.n_sink, w.window, w.gamma)
     nk = int(info["kernels"])
-    ws = binding.alloc_workspace(binding.workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, w.gamma),
-                                 dev)
+    ws = binding.alloc_workspace(binding.workspace_size(B, Hq, Hkv, N, d, w.n_sink, w.window, w.gamma), q.device)
     out = torch.empty_like(q)
     stream = torch.cuda.current_stream()
 
@@ -404,79 +464,173 @@ def run_ours(args, w, rep):
         else:
             binding.delta_attn_prefill_events(q, k, v, w.n_sink, w.window, w.gamma, evs, out=out, workspace=ws)
 
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(args.steps)]
-    for row in evs:
-        for e in row:
-            e.record(stream)  # create the events before the timed region
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         step()
     torch.cuda.synchronize()
     status = binding.check()
     if status != binding.DA_OK:
         raise RuntimeError("device status %d after warm-up" % status)
+    # length of one step, to size the number of repeats of the timed loop
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    est_ms = rep.max(e0.elapsed_time(e1))
+    repeats = max(1, min(max_repeats, int(-(-min_seconds * 1e3 // (steps * est_ms)))))
 
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(steps * repeats)]
+    for row in evs:
+        for e in row:
+            e.record(stream)  # create the events before the timed region
+    torch.cuda.synchronize()
     clocks = ClockSampler(local)
     clocks.start()
-    time.sleep(0.3)
-    rep.barrier()
-    torch.cuda.synchronize()
-    t_start = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
-    t_start.record(stream)
-    for s in range(args.steps):
-        step(evs[s])
-    t_end.record(stream)
-    torch.cuda.synchronize()
-    rep.barrier()
+    for _ in range(3):  # keep the GPU busy while the sampler starts
+        step()
+    time.sleep(0.25)
+    loop_ms = []
+    clocks.mark_start()
+    for r in range(repeats):
+        rep.barrier()
+        torch.cuda.synchronize()
+        t_start = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_start.record(stream)
+        for s in range(steps):
+            step(evs[r * steps + s])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+        rep.barrier()
+        loop_ms.append(rep.max(t_start.elapsed_time(t_end)))
+    clocks.mark_end()
     clock_info = clocks.stop()
     status = binding.check()
     if status != binding.DA_OK:
         raise RuntimeError("device status %d after the timed loop" % status)
 
-    elapsed_ms = rep.max(t_start.elapsed_time(t_end))
-    ms_per_step = elapsed_ms / args.steps
-    tokens_per_step = w.B * w.N
-    value = rep.throughput(tokens_per_step, ms_per_step / 1e3)
-
-    # per-kernel durations from the library's events (launching stream)
-    names = (["strided_dense_f32", "sink_window_fused_delta"] if nk == 2 else
-             ["strided_dense_f32", "strided_sparse_delta", "sink_window_delta"] if nk == 3 else ["dense_bf16"])
-    kt = [statistics.mean(evs[s][i].elapsed_time(evs[s][i + 1]) for s in range(args.steps)) for i in range(nk)]
-    hq_flops = 4 * w.d * w.B * w.Hq
-    dense_f = hq_flops * flops.dense_pairs_per_head(w.N, w.gamma)
-    sparse_f = hq_flops * flops.sparse_pairs_per_head(w.N, w.n_sink, w.window)
-    kflops = [dense_f, sparse_f] if nk == 2 else [dense_f, 0, sparse_f] if nk == 3 else [dense_f]
-    total_f = flops.useful_flops(w.B, w.Hq, w.N, w.d, w.n_sink, w.window, w.gamma)
+    ms_per_step = sum(loop_ms) / (repeats * steps)
+    names = KERNEL_NAMES[nk]
+    kt = [statistics.mean(row[i].elapsed_time(row[i + 1]) for row in evs) for i in range(nk)]
+    kflops = kernel_flops(w.with_(B=B, Hq=Hq, N=N, d=d), nk)
     kernels = [{"name": n, "ms": t, "share": t / sum(kt), "useful_tflops": (f / (t / 1e3) / 1e12) if f else None}
                for n, t, f in zip(names, kt, kflops)]
     dom = max(range(nk), key=lambda i: kt[i])
     peak = float(peaks.get("bf16_tflops", PEAKS_FALLBACK["bf16_tflops"]))
     achieved = kflops[dom] / (kt[dom] / 1e3) / 1e12 if kflops[dom] else None
-    traffic = recorded_traffic(names[dom], w.name)
     roofline = {"bound": "tensor", "kernel": names[dom], "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+                "frac": (achieved / peak) if achieved else None, "traffic": recorded_traffic(names[dom], w.name),
                 "peak_source": "%s bf16 dense burst (MEASURED_PEAKS.json)" % peak_src if peak_src == "measured"
                 else "fallback 1.9 PFLOP/s bf16",
                 "algorithmic": "4*d FLOPs per unmasked (query, key) pair: %.4g FLOP per launch" % kflops[dom]}
+    total_f = flops.useful_flops(B, Hq, N, d, w.n_sink, w.window, w.gamma)
     useful_tflops = total_f / (ms_per_step / 1e3) / 1e12
     sustained = float(peaks.get("bf16_tflops_sustained", PEAKS_FALLBACK["bf16_tflops_sustained"]))
+    rec = {"ms_per_step": ms_per_step, "timed_repeats": repeats, "loop_ms": loop_ms,
+           "useful_tflops": useful_tflops, "pct_of_bf16_peak": 100 * useful_tflops / peak,
+           "pct_of_bf16_sustained": 100 * useful_tflops / sustained, "roofline": roofline, "kernels": kernels,
+           "gpu_launches": nk * steps * repeats, "clocks": clock_info}
+    return rec, out, step
 
+
+def time_dense_baseline(w, q, k, v, reps, ms_delta):
+    """gamma = 1 through the same kernels: every row a dense causal row (the
+    quadratic baseline of the paper's latency figures)."""
+    from paper_2505_11254_gb300 import binding
+    stream = torch.cuda.current_stream()
+    dws = binding.alloc_workspace(binding.workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, 1),
+                                  q.device)
+    out = torch.empty_like(q)
+    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    d0.record(stream)
+    for _ in range(reps):
+        binding.delta_attn_prefill(q, k, v, w.n_sink, w.window, 1, out=out, workspace=dws)
+    d1.record(stream)
+    torch.cuda.synchronize()
+    if binding.check() != binding.DA_OK:
+        raise RuntimeError("device status after the dense baseline")
+    dense_ms = d0.elapsed_time(d1) / reps
+    dflops = flops.dense_flops(w.B, w.Hq, w.N, w.d)
+    return {"ms": dense_ms, "reps": reps, "tflops": dflops / (dense_ms / 1e3) / 1e12,
+            "speedup_of_delta": dense_ms / ms_delta,
+            "note": "gamma=1 through the same kernels = dense causal attention"}
+
+
+def time_workloads(args, dev, rep, peaks, peak_src):
+    """The million-token prefill (with its dense causal baseline) and the
+    short-window point of the B=4 sweep, through the same timed code as the
+    headline (rank 0, one GPU)."""
+    from paper_2505_11254_gb300.inputs import LLAMA8B_N1M, SWEEP_B4_N64K
+    res = {}
+    for w, dense_reps in ((LLAMA8B_N1M, 0 if args.no_dense_baseline else 1),
+                          (SWEEP_B4_N64K.with_(window=512, gamma=64), 0)):
+        q, k, v = generate(w, device=dev)
+        rec, out, _ = time_prefill(w, q, k, v, min(args.steps, 10), 3, rep, peaks, peak_src, rep.local)
+        rec.update({"tokens_per_s": w.B * w.N / (rec["ms_per_step"] / 1e3), "config": config_of(w, 1)})
+        del out
+        if dense_reps:
+            rec["dense_baseline"] = time_dense_baseline(w, q, k, v, dense_reps, rec["ms_per_step"])
+        res[w.name if w.B == 1 else "%s_w%d_g%d" % (w.name, w.window, w.gamma)] = rec
+        del q, k, v
+        torch.cuda.empty_cache()
+    return res
+
+
+def run_ours(args, w, rep):
+    from paper_2505_11254_gb300 import binding
+    from paper_2505_11254_gb300.replicas import head_shard, shard_views, gather_shards
+    world, rank, local = rep.world, rep.rank, rep.local
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    peaks, peak_src = load_peaks()
+    sharded = args.shard == "heads"
+    if sharded:
+        # one prefill, its (batch, KV head) pairs split over the ranks
+        q_all, k_all, v_all = generate(w, device=dev)
+        p0, p1 = head_shard(w.B, w.Hkv, rank, world)
+        if p1 <= p0:
+            raise RuntimeError("rank %d has no (batch, KV head) pair: use at most %d GPUs" % (rank, w.B * w.Hkv))
+        q, k, v = (t.contiguous() for t in shard_views(q_all, k_all, v_all, w.Hkv, p0, p1))
+        ws_ = w.with_(name=w.name + "_shard", B=p1 - p0, Hq=w.Hq // w.Hkv, Hkv=1)
+    else:
+        wr = w.with_(seed=rep.seed(w.seed))
+        q, k, v = generate(wr, device=dev)
+        ws_ = w
+    rec, out, step = time_prefill(ws_, q, k, v, args.steps, args.warmup, rep, peaks, peak_src, local)
+    ms_per_step = rec["ms_per_step"]
+    tokens_per_step = w.B * w.N
+    value = (tokens_per_step / (ms_per_step / 1e3)) if sharded else rep.throughput(tokens_per_step,
+                                                                                   ms_per_step / 1e3)
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "strong" if sharded else "weak",
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: seeded N(0,1) Q,K,V, RoPE base 500000 on Q,K, sink keys x%g; no dataset" % w.sink_scale,
-        "config": config_of(w, world),
-        "useful_tflops": useful_tflops, "pct_of_bf16_peak": 100 * useful_tflops / peak,
-        "pct_of_bf16_sustained": 100 * useful_tflops / sustained,
-        "roofline": roofline, "kernels": kernels, "gpu_launches": nk * args.steps,
-        "clocks": clock_info,
+        "config": config_of(w, world, args.shard),
     }
+    result.update({key: rec[key] for key in ("useful_tflops", "pct_of_bf16_peak", "pct_of_bf16_sustained",
+                                             "roofline", "kernels", "gpu_launches", "clocks", "timed_repeats",
+                                             "loop_ms")})
+    if sharded:
+        result["useful_tflops"] = flops.useful_flops(w.B, w.Hq, w.N, w.d, w.n_sink, w.window, w.gamma) / (
+            ms_per_step / 1e3) / 1e12
+        result["shard"] = {"pairs": [p0, p1], "of_pairs": w.B * w.Hkv}
+        if world > 1 and args.gather:
+            torch.cuda.synchronize()
+            rep.barrier()
+            g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            g0.record()
+            gather_shards(out, w.B, w.Hq, w.Hkv, world)
+            g1.record()
+            torch.cuda.synchronize()
+            result["shard"]["gather_ms"] = rep.max(g0.elapsed_time(g1))
 
-    if not args.no_e2e:
+    if not args.no_e2e and not sharded:
         # End to end through the C-ABI call on HOST buffers (page-locked):
         # every step copies Q, K, V in and O out; the call pipelines the
         # copies with the kernels per (batch, KV head) chunk.
+        stream = torch.cuda.current_stream()
         qh, kh, vh = (t.cpu().pin_memory() for t in (q, k, v))
         oh = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
         hws = binding.alloc_workspace(binding.host_workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window,
@@ -504,30 +658,14 @@ def run_ours(args, w, rep):
         result["e2e"]["path"] = "delta_attn_prefill_host (host buffers, copies pipelined per KV-head chunk)"
         del qh, kh, vh, oh, hws
 
-    if not args.no_dense_baseline and rank == 0:
-        # gamma = 1: every row dense, the same kernels (the paper's quadratic baseline)
-        dws = binding.alloc_workspace(binding.workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, 1), dev)
-        binding.delta_attn_prefill(q, k, v, w.n_sink, w.window, 1, out=out, workspace=dws)
-        torch.cuda.synchronize()
-        reps = 3
-        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        d0.record(stream)
-        for _ in range(reps):
-            binding.delta_attn_prefill(q, k, v, w.n_sink, w.window, 1, out=out, workspace=dws)
-        d1.record(stream)
-        torch.cuda.synchronize()
-        dense_ms = d0.elapsed_time(d1) / reps
-        dflops = flops.dense_flops(w.B, w.Hq, w.N, w.d)
-        result["dense_baseline"] = {"ms": dense_ms, "tflops": dflops / (dense_ms / 1e3) / 1e12,
-                                    "speedup_of_delta": dense_ms / ms_per_step,
-                                    "note": "gamma=1 through the same kernels = dense causal attention"}
-        del dws
-        step()  # restore `out` to the Delta result for the spot check
+    solo = rank == 0 and not sharded
+    if not args.no_dense_baseline and solo:
+        result["dense_baseline"] = time_dense_baseline(w, q, k, v, 3, ms_per_step)
 
-    if not args.no_variants and rank == 0:
-        result["variants"] = time_variants(args, w, q, k, v, out, stream, step)
+    if not args.no_variants and solo:
+        result["variants"] = time_variants(args, w, q, k, v, out, torch.cuda.current_stream(), step)
 
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if solo and world == 1 and not args.no_cpu_baseline:
         torch.cuda.synchronize()
         Qb, Kb, Vb = to_bits(q), to_bits(k), to_bits(v)
         result["parity"] = parity_spot_check(w, q, k, v, out, Qb, Kb, Vb)
@@ -537,6 +675,12 @@ def run_ours(args, w, rep):
             "sample": "%d groups of gamma=%d rows x all %d query heads at evenly spaced positions of the "
                       "%d-token sequence, fp64 C oracle on %d threads, %.1f s" % (
                           groups, w.gamma, w.Hq, w.N, cores, secs)}
+        del Qb, Kb, Vb
+
+    if solo and world == 1 and not args.no_workloads and w.name == LLAMA8B_N131K.name:
+        del q, k, v, out
+        torch.cuda.empty_cache()
+        result["workloads"] = time_workloads(args, dev, rep, peaks, peak_src)
     if rank == 0:
         print(json.dumps(result), flush=True)
 

@@ -27,8 +27,10 @@
  * validated on the host before anything is launched; invalid arguments return
  * an error and launch nothing.  Launch failures return DA_ERR_CUDA.  A kernel
  * that gives up a bounded wait (it never should) records DA_ERR_TIMEOUT in a
- * per-device status word that delta_attn_check() reports.  Results are
- * deterministic: fixed merge order, no floating-point atomics.
+ * per-device status word that delta_attn_check() reports; the word's device
+ * address is looked up once per device, on the first launching call made with
+ * that device current.  Results are deterministic: fixed merge order, no
+ * floating-point atomics.
  */
 #ifndef DELTA_ATTN_H
 #define DELTA_ATTN_H
@@ -174,9 +176,9 @@ int strided_dense_attn(const void* Q, const void* K, const void* V, float* D_sam
  * the library, held by every GPU that loads it until the process exits.  A
  * shape whose scratch (strided_dense_workspace_size()) exceeds 16 MiB returns
  * DA_ERR_WORKSPACE.  No call allocates: the first call on a device looks up
- * the array's device address (so make that first call before any stream
- * capture); every call then zeroes the scratch's tickets and counter on
- * `stream` and launches the kernel.  All calls share the one array, so calls
+ * the array's device address and the library's device status word (so make
+ * that first call before any stream capture); every call then zeroes the
+ * scratch's tickets and counter on `stream` and launches the kernel.  All calls share the one array, so calls
  * whose work overlaps on the GPU (different streams, or several host threads)
  * race and must be serialised by the caller. */
 int strided_dense_attn_noalloc(const void* Q, const void* K, const void* V, float* D_sampled, int B, int Hq,
@@ -292,8 +294,10 @@ int delta_attn_debug_rowmap(int64_t N, int gamma, int64_t* sample_row, uint8_t* 
  * 1 strided dense, 2 strided sparse) as the kernel decodes it.  out (int64,
  * device) holds 16 + 4*128 + 2*max_tiles entries: a header (b, first head,
  * kv head, first row or sample, last row or sample, sink tiles, first and last
- * band tile, tiles, chunks, chunk index, first unit, unit), then per TMEM lane
- * (row, sample, head, valid), then per key tile (tile index, needs mask). */
+ * band tile, tiles, chunks, chunk index, merge ticket, partial slot, (b, head
+ * group) index, M-tile index, split-K order: 0 longest-first, 1 key-range
+ * levels), then per TMEM lane (row, sample, head, valid), then per key tile
+ * (tile index, needs mask). */
 int delta_attn_debug_work(int mode, int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window,
                           int gamma, int64_t index, int64_t* out, int max_tiles, void* stream);
 

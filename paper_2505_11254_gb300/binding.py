@@ -358,8 +358,8 @@ def debug_work(mode, B, Hq, Hkv, N, d, n_sink, window, gamma, index, max_tiles=4
     T = hdr[8]
     return {
         "b": hdr[0], "h0": hdr[1], "g": hdr[2], "r0": hdr[3], "r_last": hdr[4], "n_sink_tiles": hdr[5],
-        "kt_lo": hdr[6], "kt_hi": hdr[7], "T": T, "n_chunks": hdr[9], "chunk_idx": hdr[10], "u0": hdr[11],
-        "unit": hdr[12],
+        "kt_lo": hdr[6], "kt_hi": hdr[7], "T": T, "n_chunks": hdr[9], "chunk_idx": hdr[10], "ticket": hdr[11],
+        "slot": hdr[12], "group": hdr[13], "mtile": hdr[14], "order": hdr[15],
         "lanes": [tuple(o[16 + 4 * t: 20 + 4 * t]) for t in range(128)],
         "tiles": [tuple(o[16 + 512 + 2 * j: 18 + 512 + 2 * j]) for j in range(min(T, max_tiles))],
     }

@@ -7,9 +7,11 @@
 
 #include <algorithm>
 #include <cmath>
+#include <mutex>
 
 #include "delta_attn.h"
 #include "launch.h"
+#include "plan.h"
 #include "tiles.cuh"
 #include "wait.cuh"
 
@@ -94,38 +96,6 @@ struct Plan {
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-// Sampled-row tiles pack Hp query heads of one KV group x R samples into the
-// 128 TMEM lanes, so the group's heads share each K/V tile.
-void packing(int G, int* Hp, int* R) {
-  int hp = 1;
-  if (G >= 2 && G <= 16 && (G & (G - 1)) == 0) hp = G;
-  *Hp = hp;
-  *R = BM / hp;
-}
-
-// Split-K plan of a strided-dense pass over p.n_s samples: the chunk is chosen
-// so that about two units per SM exist; the longest M-tiles split, short ones
-// stay whole.
-void plan_split_k(Params& p, int sms) {
-  p.mtiles = cdiv(p.n_s, p.R);
-  long long total_tiles = 0;
-  for (long long t = 0; t < p.mtiles; ++t) total_tiles += strided_dense_len(p, t);
-  total_tiles *= (long long)p.B * p.groups_per_b;
-  p.chunk = std::max<long long>(8, cdiv(total_tiles, 2LL * std::max(sms, 1)));
-  long long units = 0, multi = 0;
-  for (long long t = 0; t < p.mtiles; ++t) {
-    long long nc = cdiv(strided_dense_len(p, t), p.chunk);
-    units += nc;
-    if (nc > 1) multi += nc;
-  }
-  p.n_units = units * p.B * p.groups_per_b;
-  p.n_multi = multi * p.B * p.groups_per_b;
-}
-
-// Bytes of the control block zeroed before a strided-dense launch: 4 item
-// counters, then one merge ticket per split unit.
-size_t ctrl_bytes(const Params& p) { return 4 * sizeof(unsigned long long) + (size_t)p.n_multi * sizeof(int); }
-
 Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma, int sms,
                int64_t tail = 0, bool smooth = false) {
   Plan pl;
@@ -146,7 +116,7 @@ Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t win
   // Rows of the dense tail are recomputed densely afterwards, so the sparse
   // pass stops at the q-tile holding row N - tail - 1.
   p.qtiles = cdiv(N - tail, BM);
-  plan_split_k(p, sms);
+  plan_split_k(p, sms, d);
 
   pl.grid_sparse = (long long)B * Hq * p.qtiles;
   pl.grid_dense = p.n_units;
@@ -186,7 +156,7 @@ Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t win
     t.gamma = 1;
     t.n_s = tail;
     t.row0 = N - tail;
-    plan_split_k(t, sms);
+    plan_split_k(t, sms, d);
     pl.off_tail_part = off;
     off += align256((size_t)t.n_multi * BM * (d + 2) * sizeof(float));
     pl.off_tail_ticket = off;
@@ -199,10 +169,25 @@ Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t win
   return pl;
 }
 
+// The device address of the status word on the current device, looked up
+// once per device (with that device current) on the first call that needs it;
+// later calls only read the cached address.
+constexpr int kMaxStatusDevices = 64;
+int* g_status_addr[kMaxStatusDevices];
+cudaError_t g_status_err[kMaxStatusDevices];
+std::once_flag g_status_once[kMaxStatusDevices];
+
 int status_ptr(int** ptr) {
-  void* a = nullptr;
-  if (cudaGetSymbolAddress(&a, g_da_status) != cudaSuccess) return DA_ERR_CUDA;
-  *ptr = static_cast<int*>(a);
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return DA_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxStatusDevices) return DA_ERR_UNSUPPORTED;
+  std::call_once(g_status_once[dev], [dev] {
+    void* a = nullptr;
+    g_status_err[dev] = cudaGetSymbolAddress(&a, g_da_status);
+    g_status_addr[dev] = g_status_err[dev] == cudaSuccess ? static_cast<int*>(a) : nullptr;
+  });
+  if (g_status_err[dev] != cudaSuccess || g_status_addr[dev] == nullptr) return DA_ERR_CUDA;
+  *ptr = g_status_addr[dev];
   return DA_OK;
 }
 

@@ -823,7 +823,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       } else {
         // Dense sampled rows: the whole key range in this item, or split-K
-        // partials merged by the last CTA of the M-tile to finish.
+        // partials merged by the last CTA of the M-tile to finish (w.unit is
+        // this unit's partial slot, w.u0 the M-tile's ticket).
         const size_t slot_floats = (size_t)BM * (D + 2);
         auto store_final = [&](int q, const float* v) {
           if (EPI == EPI_DENSE_F32)
@@ -861,14 +862,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           named_bar_sync(2, 128);  // ticket_sh is rewritten by the next split item
           if (merge && row_ok) {
             __threadfence();
+            // Branch-free over the chunks, unrolled so that several partials'
+            // loads are in flight at once.  A chunk no key of which this row
+            // sees has m = -inf, l = 0 and O = 0: its weight is 0.
             float mstar = -INFINITY;
+#pragma unroll 4
             for (int c = 0; c < w.n_chunks; ++c)
-              mstar = fmaxf(mstar, __ldcg(p.partials + (size_t)(w.u0 + c) * slot_floats + (size_t)BM * D + e));
+              mstar = fmaxf(mstar, __ldcg(p.partials + (size_t)partial_slot(p, w, c) * slot_floats + (size_t)BM * D + e));
             float lsum = 0.f;
+#pragma unroll 4
             for (int c = 0; c < w.n_chunks; ++c) {
-              const float* pc = p.partials + (size_t)(w.u0 + c) * slot_floats;
+              const float* pc = p.partials + (size_t)partial_slot(p, w, c) * slot_floats;
               const float mc = __ldcg(pc + (size_t)BM * D + e);
-              if (mc != -INFINITY) lsum += __ldcg(pc + (size_t)BM * D + BM + e) * ex2(mc - mstar);
+              const float lc = __ldcg(pc + (size_t)BM * D + BM + e);
+              lsum += (mc == -INFINITY) ? 0.f : lc * ex2(mc - mstar);
             }
             const float inv = (lsum > 0.f) ? 1.f / lsum : 0.f;
 #pragma unroll 1
@@ -876,15 +883,15 @@ __global__ void __launch_bounds__(kThreads, 1)
               float v[32];
 #pragma unroll
               for (int c = 0; c < 32; ++c) v[c] = 0.f;
+#pragma unroll 2
               for (int c2 = 0; c2 < w.n_chunks; ++c2) {
-                const float* pc = p.partials + (size_t)(w.u0 + c2) * slot_floats;
+                const float* pc = p.partials + (size_t)partial_slot(p, w, c2) * slot_floats;
                 const float mc = __ldcg(pc + (size_t)BM * D + e);
-                if (mc == -INFINITY) continue;
-                const float f = ex2(mc - mstar);
                 float x[32];
                 load_f32x32_cg(pc + (size_t)e * D + q * 32, x);
+                const float f = (mc == -INFINITY) ? 0.f : ex2(mc - mstar);
 #pragma unroll
-                for (int c = 0; c < 32; ++c) v[c] += x[c] * f;
+                for (int c = 0; c < 32; ++c) v[c] = fmaf(x[c], f, v[c]);
               }
 #pragma unroll
               for (int c = 0; c < 32; ++c) v[c] *= inv;

@@ -125,7 +125,7 @@ __device__ void debug_work_body(const Params& p, long long index, long long* out
   const int t = threadIdx.x;
   if (t == 0) {
     long long h[16] = {w.b, w.h0, w.g, w.r0, w.r_last, w.n_sink_tiles, w.kt_lo, w.kt_hi,
-                       w.T, w.n_chunks, w.chunk_idx, w.u0, w.unit, 0, 0, 0};
+                       w.T, w.n_chunks, w.chunk_idx, w.u0, w.unit, w.gi, w.t, p.order};
     for (int e = 0; e < 16; ++e) out[e] = h[e];
   }
   if (t < BM) {

@@ -44,6 +44,13 @@ enum Smooth : int {
 };
 constexpr int kSmoothJ = 2;  // basis vectors per sample (the filter uses the first)
 
+// Order of the strided dense pass's split-K units (plan.h).
+enum SplitOrder : int {
+  SPLIT_LONGEST_FIRST = 0,  // M-tiles by descending t, each cut into chunks
+  SPLIT_LEVELS = 1,         // head group by head group, key-range levels from the top, t descending
+};
+constexpr int kMaxLevels = 32;
+
 struct Params {
   int B, Hq, Hkv, G;
   long long N;
@@ -59,9 +66,14 @@ struct Params {
   long long mtiles;        // ceil(n_s / R) tiles per head group
   long long qtiles;        // ceil(N / BM) tiles of contiguous rows per head
   // split-K over keys for MODE_STRIDED_DENSE
+  int order;               // SplitOrder
+  int n_lev;               // SPLIT_LEVELS: key-range levels of `chunk` tiles
   long long chunk;         // key tiles per unit
-  long long n_units;       // units (= CTAs)
-  long long n_multi;       // leading units that belong to split M-tiles
+  long long n_units;       // units
+  long long n_multi;       // units of split M-tiles (partial slots)
+  long long units_per_group;   // SPLIT_LEVELS: units of one (b, head group)
+  long long split_per_group;   // SPLIT_LEVELS: of which belong to split M-tiles (the group's first units)
+  long long lev_cum[kMaxLevels + 1];  // SPLIT_LEVELS: units of a group before step l (level n_lev - 1 - l)
   long long n_items;       // work items of the launched kernel
   // buffers
   void* out_bf16;          // [B,Hq,N,d] bf16
@@ -87,7 +99,9 @@ struct Work {
   long long kt_lo;     // band tiles [kt_lo, kt_hi]
   long long kt_hi;
   int T;               // number of key tiles visited
-  long long unit, u0;  // split-K: this unit, first unit of its M-tile
+  long long unit;      // split-K: this unit's partial slot (when its M-tile is split)
+  long long u0;        // split-K: merge ticket of its M-tile
+  long long gi, t;     // split-K: (b, head group) index and M-tile index
   int chunk_idx, n_chunks;
 };
 
@@ -117,22 +131,76 @@ __host__ __device__ __forceinline__ long long strided_dense_len(const Params& p,
   return (p.row0 + k_last * p.gamma) / BN + 1;
 }
 
-// Split-K units are ordered longest-first: M-tile index t descending, then
-// (b, head group), then chunk.  Units of M-tiles with more than one chunk come
-// first because the chunk count never decreases with t.
+// lev_cum[l] for a run-time l, read with constant indices only (the
+// parameter block is never indexed dynamically).
+__host__ __device__ __forceinline__ long long lev_cum_at(const Params& p, int l) {
+  long long v = 0;
+#pragma unroll
+  for (int i = 0; i <= kMaxLevels; ++i)
+    if (i == l) v = p.lev_cum[i];
+  return v;
+}
+
+// Partial slot of chunk c of the unit's M-tile (its units hold the chunks
+// 0 .. n_chunks - 1).
+__host__ __device__ __forceinline__ long long partial_slot(const Params& p, const Work& w, int c) {
+  if (p.order == SPLIT_LEVELS)
+    return w.gi * p.split_per_group + lev_cum_at(p, p.n_lev - 1 - c) + (p.mtiles - 1 - w.t);
+  return w.u0 + c;
+}
+
+// Split-K units, in the order of p.order (plan.h):
+//   SPLIT_LONGEST_FIRST: M-tile index t descending, then (b, head group), then
+//     chunk.  Units of M-tiles with more than one chunk come first because the
+//     chunk count never decreases with t; a unit's partial slot is its index,
+//     its M-tile's ticket the index of its first chunk.
+//   SPLIT_LEVELS: (b, head group) outermost; inside a group, level c from
+//     n_lev - 1 down to 0 (key tiles [c chunk, (c+1) chunk)), inside a level
+//     the M-tiles long enough to reach it by descending t.  The units of
+//     split M-tiles are the first split_per_group of each group, which gives
+//     their partial slots; the ticket is the slot of the level-0 unit.
 __host__ __device__ inline Work decode_strided_dense(const Params& p, long long unit) {
   Work w;
-  long long per_t = (long long)p.B * p.groups_per_b;
-  long long cum = 0, t = p.mtiles - 1, nc = 1;
-  for (; t >= 0; --t) {
+  long long t, nc, mt;
+  int c;
+  if (p.order == SPLIT_LEVELS) {
+    const long long gi = unit / p.units_per_group;
+    const long long ul = unit - gi * p.units_per_group;
+    int l = 0;
+    long long base = 0;
+#pragma unroll
+    for (int i = 1; i < kMaxLevels; ++i)
+      if (i < p.n_lev && p.lev_cum[i] <= ul) {
+        l = i;
+        base = p.lev_cum[i];
+      }
+    c = p.n_lev - 1 - l;
+    t = p.mtiles - 1 - (ul - base);
     nc = cdiv(strided_dense_len(p, t), p.chunk);
-    if (unit < cum + nc * per_t) break;
-    cum += nc * per_t;
+    mt = gi;
+    w.gi = gi;
+    w.t = t;
+    w.unit = gi * p.split_per_group + ul;
+    w.u0 = gi * p.split_per_group + lev_cum_at(p, p.n_lev - 1) + (p.mtiles - 1 - t);
+  } else {
+    long long per_t = (long long)p.B * p.groups_per_b;
+    long long cum = 0;
+    t = p.mtiles - 1;
+    nc = 1;
+    for (; t >= 0; --t) {
+      nc = cdiv(strided_dense_len(p, t), p.chunk);
+      if (unit < cum + nc * per_t) break;
+      cum += nc * per_t;
+    }
+    if (t < 0) t = 0;  // unreachable for unit < n_units
+    long long rem = unit - cum;
+    mt = rem / nc;
+    c = (int)(rem % nc);
+    w.gi = mt;
+    w.t = t;
+    w.unit = unit;
+    w.u0 = unit - c;
   }
-  if (t < 0) t = 0;  // unreachable for unit < n_units
-  long long rem = unit - cum;
-  long long mt = rem / nc;
-  int c = (int)(rem % nc);
   w.b = (int)(mt / p.groups_per_b);
   int hg = (int)(mt % p.groups_per_b);
   w.h0 = hg * p.Hp;
@@ -144,8 +212,6 @@ __host__ __device__ inline Work decode_strided_dense(const Params& p, long long 
   w.kt_lo = (long long)c * p.chunk;
   w.kt_hi = lmin(L, (long long)(c + 1) * p.chunk) - 1;
   w.T = (int)(w.kt_hi - w.kt_lo + 1);
-  w.unit = unit;
-  w.u0 = unit - c;
   w.chunk_idx = c;
   w.n_chunks = (int)nc;
   return w;
@@ -184,7 +250,7 @@ __host__ __device__ inline Work decode_sparse(const Params& p, long long lin) {
   w.kt_hi = w.r_last / BN;
   w.n_sink_tiles = sink_tiles_before(p.n_sink, w.r_last, w.kt_lo);
   w.T = w.n_sink_tiles + (int)(w.kt_hi - w.kt_lo + 1);
-  w.unit = w.u0 = 0;
+  w.unit = w.u0 = w.gi = w.t = 0;
   w.chunk_idx = 0;
   w.n_chunks = 1;
   return w;
@@ -206,7 +272,7 @@ __host__ __device__ inline Work decode_strided_sparse(const Params& p, long long
   w.kt_hi = row_last / BN;
   w.n_sink_tiles = sink_tiles_before(p.n_sink, row_last, w.kt_lo);
   w.T = w.n_sink_tiles + (int)(w.kt_hi - w.kt_lo + 1);
-  w.unit = w.u0 = 0;
+  w.unit = w.u0 = w.gi = w.t = 0;
   w.chunk_idx = 0;
   w.n_chunks = 1;
   return w;

@@ -1,11 +1,14 @@
-"""Data-parallel replicas of the Delta Attention prefill across GPUs.
+"""Data-parallel replicas and head shards of the Delta Attention prefill
+across GPUs.
 
 The prefill partitions into independent problems (sequences; (batch, KV head)
-groups with their query heads) with no exchange, so N GPUs run N independent
-problems: one process per GPU (launched by torchrun), each with its own seeded
-sequence, and no collective on the data path.  Timing uses a barrier on both
-sides of the timed loop and the maximum of the per-rank times; whole-job
-throughput is the total work of all ranks over that time (weak scaling).
+groups with their query heads) with no exchange.  Two ways to use N GPUs, one
+process per GPU (launched by torchrun), no collective on the data path:
+  * replicas: N independent seeded sequences, one per rank (weak scaling);
+  * head shards: one prefill whose (batch, KV head) pairs are split over the
+    ranks (strong scaling), optionally followed by an all-gather of O.
+Timing uses a barrier on both sides of the timed loop and the maximum of the
+per-rank times; whole-job throughput is the work of all ranks over that time.
 
 Works with NCCL on GPUs and with gloo on CPU (used by the host-side tests).
 """
@@ -64,3 +67,51 @@ class Replicas:
             import torch.distributed as dist
             if dist.is_initialized():
                 dist.destroy_process_group()
+
+
+# ---------------------------------------------------------------- head shards
+# One prefill split over ranks.  The (batch, KV head) pairs of Alg. 1 are
+# independent problems (each query head reads only its own KV head), so rank r
+# takes a contiguous range of the B * Hkv pairs with the G query heads of each
+# pair and runs the unchanged single-GPU path on it, with no exchange on the
+# data path.  In the [B * Hkv, G, N, d] view of Q and O (and [B * Hkv, 1, N, d]
+# of K and V) a contiguous pair range is one contiguous slice, which the
+# library takes as a problem of (p1 - p0) sequences with G query heads and one
+# KV head.
+
+def head_shard(B: int, Hkv: int, rank: int, world: int):
+    """Pair range [p0, p1) of rank `rank`: the B * Hkv pairs split into
+    `world` contiguous ranges whose sizes differ by at most one."""
+    if world < 1 or not 0 <= rank < world:
+        raise ValueError("rank %d outside a world of %d" % (rank, world))
+    pairs = B * Hkv
+    return rank * pairs // world, (rank + 1) * pairs // world
+
+
+def shard_views(Q, K, V, Hkv: int, p0: int, p1: int):
+    """Views of Q [B, Hq, N, d] and K, V [B, Hkv, N, d] holding the pairs
+    [p0, p1): Q as [p1 - p0, G, N, d], K and V as [p1 - p0, 1, N, d]."""
+    B, Hq, N, d = Q.shape
+    G = Hq // Hkv
+    q = Q.reshape(B * Hkv, G, N, d)[p0:p1]
+    k = K.reshape(B * Hkv, 1, N, d)[p0:p1]
+    v = V.reshape(B * Hkv, 1, N, d)[p0:p1]
+    return q, k, v
+
+
+def gather_shards(O_part, B: int, Hq: int, Hkv: int, world: int):
+    """All-gather of the per-rank outputs O_part [p1 - p0, G, N, d] into the
+    whole [B, Hq, N, d] output (every rank receives it).  Shards are padded to
+    the largest range so that the collective moves equal-sized buffers."""
+    import torch.distributed as dist
+    G, N, d = O_part.shape[1:]
+    ranges = [head_shard(B, Hkv, r, world) for r in range(world)]
+    width = max(p1 - p0 for p0, p1 in ranges)
+    pad = O_part.new_zeros((width, G, N, d))
+    pad[: O_part.shape[0]].copy_(O_part)
+    bufs = [torch.empty_like(pad) for _ in range(world)]
+    dist.all_gather(bufs, pad)
+    out = O_part.new_empty((B * Hkv, G, N, d))
+    for (p0, p1), buf in zip(ranges, bufs):
+        out[p0:p1].copy_(buf[: p1 - p0])
+    return out.reshape(B, Hq, N, d)

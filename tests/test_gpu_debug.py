@@ -58,26 +58,39 @@ def test_sparse_tiles_cover_exactly_the_sparse_set(shape):
 
 @pytest.mark.parametrize("shape", SHAPES + [(1, 32, 8, 131072, 128, 4, 2048, 64)])
 def test_dense_units_partition_the_causal_range(shape):
+    """The device decode of the split-K units: each M-tile's chunks tile its
+    causal key range [0, last causal key] exactly once, split M-tiles' chunks
+    hold distinct partial slots and share one ticket (checked for every M-tile
+    whose chunks are all among the units read: all units up to 6000)."""
     B, Hq, Hkv, N, d, s, w, gamma = shape
     info = binding.plan_info(*shape)
     ns = n_samples(N, gamma)
-    covered = {}
-    for u in range(info["ctas_dense"]):
+    chunks, slots, tickets = {}, set(), {}
+    for u in range(min(info["ctas_dense"], 6000)):
         wk = binding.debug_work(1, *shape, u)
         key = (wk["b"], wk["h0"], wk["r0"])
         tiles = [t for t, _ in wk["tiles"]]
-        covered.setdefault(key, []).extend(tiles)
+        assert wk["chunk_idx"] not in chunks.setdefault(key, {}), "a chunk is held twice"
+        chunks[key][wk["chunk_idx"]] = (wk["n_chunks"], tiles)
+        if wk["n_chunks"] > 1:
+            assert 0 <= wk["slot"] < info["split_units"] and wk["slot"] not in slots, "partial slot"
+            slots.add(wk["slot"])
+            assert tickets.setdefault(key, wk["ticket"]) == wk["ticket"], "one ticket per M-tile"
         lanes = [(row, smp, h) for (row, smp, h, ok) in wk["lanes"] if ok]
         assert lanes and max(r for r, _, _ in lanes) <= (ns - 1) * gamma
         assert all(r == smp * gamma for r, smp, _ in lanes)
         for t, masked in wk["tiles"]:
             if not masked:
                 assert t * 128 + 127 <= min(r for r, _, _ in lanes)
-        if len(covered) > 400:
-            del covered[key]  # possibly incomplete: its other units were not read
-            break
     R = info["samples_per_head"]
-    for (b, h0, k0), tiles in covered.items():
-        # each M-tile's units tile [0, last causal key] exactly once
+    complete = 0
+    for (b, h0, k0), got in chunks.items():
+        n_chunks = next(iter(got.values()))[0]
+        if len(got) < n_chunks:
+            continue  # some of its units were not read
+        complete += 1
+        tiles = sorted(t for c in got.values() for t in c[1])
         k_last = min(k0 + R - 1, ns - 1)
-        assert sorted(tiles) == list(range(k_last * gamma // 128 + 1))
+        assert tiles == list(range(k_last * gamma // 128 + 1))
+    assert complete > 0
+    assert len(set(tickets.values())) == len(tickets), "M-tiles share a ticket"

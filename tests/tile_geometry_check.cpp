@@ -3,9 +3,9 @@
 // three modes, unmasked_tiles() must select exactly the tiles for which
 // tile_needs_mask() is false, and tile_needs_mask() must be true wherever a
 // (row, key) pair of the tile is not visible (checked pair by pair against
-// the definition of the key sets), and the dense pass's split-K units cover
-// every M-tile's causal key range exactly once in the order the partial slots
-// and tickets assume.  For every head packing of the dense tiles (GQA 1, 2,
+// the definition of the key sets), and the dense pass's split-K units, as the
+// library's planner (plan.h) lays them out, cover every M-tile's causal key
+// range exactly once with the partial slots and tickets the merge assumes.  For every head packing of the dense tiles (GQA 1, 2,
 // 3, 4 and 16), each lane's query head reads its own KV head (floor(h / G))
 // and every (batch, head, row or sample) sits in exactly one lane.
 #define __host__
@@ -15,6 +15,7 @@
 #include <cstdlib>
 #include <initializer_list>
 #include <vector>
+#include "plan.h"
 #include "tiles.cuh"
 
 using namespace da;
@@ -88,84 +89,141 @@ static int check(const Params& p, long long items) {
   return bad;
 }
 
-// The split-K units of the dense pass: every M-tile's key range [0, L) is
-// covered exactly once by adjacent units u0 .. u0 + n_chunks - 1, units with
-// more than one chunk are exactly [0, n_multi), and the (b, head group, t)
-// of each unit is a valid M-tile.
+// The split-K units of the dense pass, for a plan made by plan_split_k():
+// every M-tile's causal key range [0, L) is covered exactly once by its chunks
+// (chunk c holds tiles [c chunk, min(L, (c+1) chunk))); the units of split
+// M-tiles hold distinct partial slots that fill [0, n_multi), and
+// partial_slot() finds every chunk's slot; each split M-tile has one merge
+// ticket, distinct from every other M-tile's, in [0, n_multi); the unit's
+// (b, head group) and M-tile index are those of its rows.  In the level
+// order, units run group by group, level by level from the top, and by
+// descending M-tile inside a level, each at most `chunk` tiles.
 static int check_dense_units(const Params& p) {
   int bad = 0;
-  std::vector<long long> cover((size_t)p.B * p.groups_per_b * p.mtiles, -1);
-  std::vector<int> seen_tiles((size_t)p.B * p.groups_per_b * p.mtiles, 0);
+  auto fail = [&](const char* what, long long u) {
+    if (bad < 5) std::printf("dense unit %lld (order %d): %s\n", u, p.order, what);
+    ++bad;
+  };
+  const long long n_mt = (long long)p.B * p.groups_per_b * p.mtiles;
+  std::vector<long long> covered((size_t)n_mt, 0), ticket_of((size_t)n_mt, -1);
+  std::vector<std::vector<long long>> slot_of_chunk((size_t)n_mt);
+  std::vector<char> slot_used((size_t)p.n_multi, 0), ticket_used((size_t)p.n_multi, 0);
+  long long prev_gi = -1, prev_c = 0, prev_t = 0;
   for (long long u = 0; u < p.n_units; ++u) {
     const Work w = decode_strided_dense(p, u);
     const long long t = w.r0 / p.R;
-    const long long idx = ((long long)w.b * p.groups_per_b + w.h0 / p.Hp) * p.mtiles + t;
+    const long long gi = (long long)w.b * p.groups_per_b + w.h0 / p.Hp;
+    if (w.b < 0 || w.b >= p.B || t < 0 || t >= p.mtiles || w.t != t || w.gi != gi) {
+      fail("rows do not match the M-tile index", u);
+      continue;
+    }
+    const long long idx = gi * p.mtiles + t;
     const long long L = strided_dense_len(p, t);
-    bool ok = w.b >= 0 && w.b < p.B && t >= 0 && t < p.mtiles && w.kt_lo == (long long)w.chunk_idx * p.chunk &&
-              w.kt_hi == lmin(L, (long long)(w.chunk_idx + 1) * p.chunk) - 1 && w.n_chunks == cdiv(L, p.chunk) &&
-              w.u0 == u - w.chunk_idx && ((w.n_chunks > 1) == (u < p.n_multi));
-    if (ok && w.chunk_idx == 0) {
-      ok = cover[idx] < 0;
-      cover[idx] = u;
+    const int c = w.chunk_idx;
+    if (w.kt_lo != (long long)c * p.chunk || w.kt_hi != lmin(L, (long long)(c + 1) * p.chunk) - 1 ||
+        w.n_chunks != cdiv(L, p.chunk) || w.T != w.kt_hi - w.kt_lo + 1 || w.T < 1)
+      fail("key range of the chunk", u);
+    std::vector<long long>& sl = slot_of_chunk[(size_t)idx];
+    if (sl.empty()) sl.assign((size_t)w.n_chunks, -2);
+    if (c < 0 || c >= (int)sl.size() || sl[(size_t)c] != -2) {
+      fail("chunk held twice", u);
+      continue;
     }
-    if (ok) seen_tiles[idx] += w.T;
+    sl[(size_t)c] = w.unit;
+    covered[(size_t)idx] += w.T;
+    if (w.n_chunks > 1) {
+      if (w.unit < 0 || w.unit >= p.n_multi || slot_used[(size_t)w.unit]) fail("partial slot", u);
+      else slot_used[(size_t)w.unit] = 1;
+      if (partial_slot(p, w, c) != w.unit) fail("partial_slot() of its own chunk", u);
+      if (w.u0 < 0 || w.u0 >= p.n_multi) fail("ticket out of range", u);
+      else if (ticket_of[(size_t)idx] < 0) {
+        if (ticket_used[(size_t)w.u0]) fail("ticket shared by two M-tiles", u);
+        ticket_used[(size_t)w.u0] = 1;
+        ticket_of[(size_t)idx] = w.u0;
+      } else if (ticket_of[(size_t)idx] != w.u0) {
+        fail("chunks of one M-tile with different tickets", u);
+      }
+    }
+    if (p.order == SPLIT_LEVELS) {
+      if (w.T > p.chunk) fail("unit longer than a chunk", u);
+      const bool next = gi > prev_gi || (gi == prev_gi && (c < prev_c || (c == prev_c && t < prev_t)));
+      if (u > 0 && !next) fail("level order", u);
+      if (gi < prev_gi) fail("group order", u);
+      prev_gi = gi;
+      prev_c = c;
+      prev_t = t;
+    }
+  }
+  for (long long idx = 0; idx < n_mt; ++idx) {
+    const long long t = idx % p.mtiles;
+    const std::vector<long long>& sl = slot_of_chunk[(size_t)idx];
+    bool ok = covered[(size_t)idx] == strided_dense_len(p, t) && !sl.empty();
+    for (size_t c = 0; ok && c < sl.size(); ++c) ok = sl[c] != -2;
+    if (ok && sl.size() > 1) {  // the merge finds every chunk's partial from any unit of the M-tile
+      const Work w = decode_strided_dense(p, 0);
+      Work m = w;
+      m.gi = idx / p.mtiles;
+      m.t = t;
+      m.u0 = ticket_of[(size_t)idx];
+      for (size_t c = 0; ok && c < sl.size(); ++c) ok = partial_slot(p, m, (int)c) == sl[c];
+    }
     if (!ok) {
-      if (bad < 5) std::printf("dense unit %lld: bad decode (t %lld chunk %d of %d)\n", u, t, w.chunk_idx, w.n_chunks);
+      if (bad < 5) std::printf("dense M-tile %lld (order %d) not covered exactly once\n", idx, p.order);
       ++bad;
     }
   }
-  for (size_t i = 0; i < cover.size(); ++i) {
-    const long long t = (long long)(i % p.mtiles);
-    if (cover[i] < 0 || seen_tiles[i] != strided_dense_len(p, t)) {
-      if (bad < 5) std::printf("dense M-tile %zu not covered exactly once\n", i);
+  for (long long sidx = 0; sidx < p.n_multi; ++sidx)
+    if (!slot_used[(size_t)sidx]) {
+      if (bad < 5) std::printf("partial slot %lld (order %d) unused\n", sidx, p.order);
       ++bad;
     }
-  }
   return bad;
 }
 
-// Hp query heads of one KV group share a dense tile when G is a power of two
-// up to 16 (R = 128 / Hp samples each); otherwise one head per tile.
-static void set_packing(Params& p) {
-  p.Hp = (p.G >= 2 && p.G <= 16 && (p.G & (p.G - 1)) == 0) ? p.G : 1;
-  p.R = BM / p.Hp;
-  p.groups_per_b = p.Hq / p.Hp;
-}
-
-static long long count_units(Params& p) {
-  p.mtiles = (p.n_s + p.R - 1) / p.R;
-  long long units = 0, multi = 0;
-  for (long long t = 0; t < p.mtiles; ++t) {
-    const long long nc = (strided_dense_len(p, t) + p.chunk - 1) / p.chunk;
-    units += nc;
-    if (nc > 1) multi += nc;
-  }
-  p.n_units = units * p.B * p.groups_per_b;
-  p.n_multi = multi * p.B * p.groups_per_b;
-  return p.n_units;
-}
+// Plans made by the library's planner for several machines and policies:
+// SM counts 152, 7 and 1; the library's policy; units of a few tiles (many
+// levels on small shapes); at most two levels; and a zero budget
+// (longest-first whenever an M-tile splits).
+struct PlanCase {
+  int sms;
+  SplitPolicy pol;
+};
+static const PlanCase kPlans[] = {{152, {kMaxLevelsUsed, kUnitTiles, kMinChunk, kLevelPartialBytes}},
+                                  {7, {kMaxLevelsUsed, 2, 1, kLevelPartialBytes}},
+                                  {1, {2, 1, 1, kLevelPartialBytes}},
+                                  {152, {kMaxLevelsUsed, 3, 1, 0}},
+                                  {1, {kMaxLevels, 1, 1, kLevelPartialBytes}}};
 
 static int check_shape(int B, int Hq, int Hkv, long long N, long long win, int ns, int gm) {
   int bad = 0;
   Params p = {};
   p.B = B; p.Hq = Hq; p.Hkv = Hkv; p.G = Hq / Hkv; p.N = N; p.n_sink = ns; p.window = win; p.gamma = gm;
   p.n_s = (N + gm - 1) / gm;
-  set_packing(p);
+  packing(p.G, &p.Hp, &p.R);
+  p.groups_per_b = p.Hq / p.Hp;
   p.qtiles = (N + BM - 1) / BM;
-  p.chunk = 3;
-  count_units(p);
+  plan_split_k(p, 152, 128);
   bad += check<MODE_SPARSE>(p, (long long)p.B * p.Hq * p.qtiles);
   bad += check<MODE_STRIDED_SPARSE>(p, (long long)p.B * p.groups_per_b * p.mtiles);
-  bad += check<MODE_STRIDED_DENSE>(p, p.n_units);
-  bad += check_dense_units(p);
-  // the dense tail: gamma 1 from row N - tail
-  for (long long tail : {1LL, 77LL, N}) {
-    if (tail > N) continue;
+  {  // the library's own policy for this shape
     Params q = p;
-    q.gamma = 1; q.n_s = tail; q.row0 = N - tail;
-    count_units(q);
+    plan_split_k(q, 152, 128);
+    bad += check_dense_units(q);
+  }
+  for (const PlanCase& pc : kPlans) {
+    Params q = p;
+    plan_split_k(q, pc.sms, 128, pc.pol);
     bad += check<MODE_STRIDED_DENSE>(q, q.n_units);
     bad += check_dense_units(q);
+    // the dense tail: gamma 1 from row N - tail
+    for (long long tail : {1LL, 77LL, N}) {
+      if (tail > N) continue;
+      Params r = p;
+      r.gamma = 1; r.n_s = tail; r.row0 = N - tail;
+      plan_split_k(r, pc.sms, 128, pc.pol);
+      bad += check<MODE_STRIDED_DENSE>(r, r.n_units);
+      bad += check_dense_units(r);
+    }
   }
   return bad;
 }
