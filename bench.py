@@ -19,9 +19,9 @@ dense kernel, then the sink+window kernel with the fused Delta epilogue.
                  (appendix "Implementation Details") and the three Delta
                  smoothing forms (appendix "Interpolation"), timed the same way
 
-  workloads      (default workload only) the million-token prefill with its
-                 dense baseline, and the B=4 sweep's window-512 gamma-64 point,
-                 through the same timed code
+  workloads      (default workload only) the 32K layer and the million-token
+                 prefill, each with its dense baseline, and the twelve points of
+                 the B=4 window/gamma sweep, through the same timed code
 
 The timed loop of --steps prefills is repeated back to back until the timed
 region lasts about one second (each repeat bracketed by a barrier and a
@@ -57,7 +57,7 @@ from paper_2505_11254_gb300.inputs import WORKLOADS, LLAMA8B_N131K, generate, to
 METRIC = "Δ-attn prefill tokens/s and useful TFLOP/s (% bf16 tensor peak) at N=131K/1M"
 UNIT = "tokens/s"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-KERNEL_SOURCES = ["attn_kernel.cuh", "tiles.cuh", "ptx.cuh", "wait.cuh", "launch_impl.cuh"]
+KERNEL_SOURCES = ["attn_kernel.cuh", "tiles.cuh", "plan.h", "ptx.cuh", "wait.cuh", "launch_impl.cuh"]
 
 
 def parse_args():
@@ -76,7 +76,7 @@ def parse_args():
     ap.add_argument("--no-variants", action="store_true", help="skip the Eq. 5 / dense-tail timings")
     ap.add_argument("--tail", type=int, default=1024, help="dense tail rows of the variant timings")
     ap.add_argument("--no-workloads", action="store_true",
-                    help="skip the 1M-token and B=4 window-512 records of the default run")
+                    help="skip the records of the other configurations (32K, 1M, the B=4 sweep)")
     ap.add_argument("--shard", choices=["replicas", "heads"], default="replicas",
                     help="N GPUs: independent sequences (weak scaling) or one prefill split by (batch, KV head) "
                          "pairs (strong scaling)")
@@ -557,22 +557,37 @@ def time_dense_baseline(w, q, k, v, reps, ms_delta):
 
 
 def time_workloads(args, dev, rep, peaks, peak_src):
-    """The million-token prefill (with its dense causal baseline) and the
-    short-window point of the B=4 sweep, through the same timed code as the
-    headline (rank 0, one GPU)."""
-    from paper_2505_11254_gb300.inputs import LLAMA8B_N1M, SWEEP_B4_N64K
+    """The other configurations, through the same timed code as the headline
+    (rank 0, one GPU): the 32K layer, the million-token prefill with its
+    dense causal baseline, and the twelve points of the B=4 window/gamma sweep
+    (one set of inputs; window and gamma change only the kernels' work)."""
+    from paper_2505_11254_gb300.inputs import LLAMA8B_N1M, LLAMA8B_N32K, SWEEP_B4_N64K, SWEEP_GAMMAS, SWEEP_WINDOWS
     res = {}
-    for w, dense_reps in ((LLAMA8B_N1M, 0 if args.no_dense_baseline else 1),
-                          (SWEEP_B4_N64K.with_(window=512, gamma=64), 0)):
-        q, k, v = generate(w, device=dev)
+
+    def one(w, q, k, v, dense_reps=0):
         rec, out, _ = time_prefill(w, q, k, v, min(args.steps, 10), 3, rep, peaks, peak_src, rep.local)
         rec.update({"tokens_per_s": w.B * w.N / (rec["ms_per_step"] / 1e3), "config": config_of(w, 1)})
+        for key in ("loop_ms",):
+            rec.pop(key, None)
         del out
         if dense_reps:
             rec["dense_baseline"] = time_dense_baseline(w, q, k, v, dense_reps, rec["ms_per_step"])
-        res[w.name if w.B == 1 else "%s_w%d_g%d" % (w.name, w.window, w.gamma)] = rec
+        return rec
+
+    for w, dense_reps in ((LLAMA8B_N32K, 0 if args.no_dense_baseline else 3),
+                          (LLAMA8B_N1M, 0 if args.no_dense_baseline else 1)):
+        q, k, v = generate(w, device=dev)
+        res[w.name] = one(w, q, k, v, dense_reps)
         del q, k, v
         torch.cuda.empty_cache()
+    q, k, v = generate(SWEEP_B4_N64K, device=dev)
+    sweep = {}
+    for window in SWEEP_WINDOWS:
+        for gamma in SWEEP_GAMMAS:
+            sweep["w%d_g%d" % (window, gamma)] = one(SWEEP_B4_N64K.with_(window=window, gamma=gamma), q, k, v)
+    res[SWEEP_B4_N64K.name] = sweep
+    del q, k, v
+    torch.cuda.empty_cache()
     return res
 
 

@@ -117,6 +117,20 @@ __host__ __device__ __forceinline__ bool visible_sparse(long long i, long long j
 __host__ __device__ __forceinline__ long long sample_of_row(long long i, int gamma) { return (i / gamma) * gamma; }
 __host__ __device__ __forceinline__ bool is_sampled_row(long long i, int gamma) { return i % gamma == 0; }
 
+// Visibility word of the key offsets c0 .. c0 + 31 of a tile: bit c - c0 is
+// set when lo <= c <= hi (window and causality; hi < lo is an empty range) or
+// c < se (sinks).  The kernels mask a tile's scores by one bit test per key.
+__host__ __device__ __forceinline__ uint32_t visible_bits(int lo, int hi, int se, int c0) {
+  const int a = lo - c0 > 0 ? lo - c0 : 0;
+  const int b = hi - c0 < 31 ? hi - c0 : 31;
+  const uint32_t upto_b = b < 0 ? 0u : (b >= 31 ? 0xffffffffu : ((2u << b) - 1u));
+  const uint32_t below_a = a >= 32 ? 0xffffffffu : ((1u << a) - 1u);
+  const uint32_t range = b >= a ? (upto_b & ~below_a) : 0u;
+  const int ns = se - c0 < 0 ? 0 : (se - c0 > 32 ? 32 : se - c0);
+  const uint32_t sink = ns >= 32 ? 0xffffffffu : ((1u << ns) - 1u);
+  return range | sink;
+}
+
 // Key tiles covering the sink keys visible to rows up to `last_row`, limited
 // to tiles before the band's first tile.
 __host__ __device__ __forceinline__ int sink_tiles_before(int n_sink, long long last_row, long long kt_lo) {

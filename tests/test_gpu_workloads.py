@@ -13,7 +13,8 @@ oracle on sets of output rows, each set with its own max-abs and mean-abs:
   early    rows 1, 2, 3, 5, 9, 17: dominated by the sink keys (scaled x8 at
            131K)
 
-for four (b, h) pairs on distinct KV heads (and distinct sequences for B=4).
+for four (b, h) pairs on distinct KV heads (and distinct sequences for B=4);
+the small 2048-token configuration is compared on every element.
 Tolerance: max-abs 2e-2, mean-abs 2e-3 per set.  With DA_PARITY_RECORD set to
 a file name, every set's figures are appended to it as JSON lines.
 """
@@ -27,7 +28,7 @@ import torch
 import oracle
 from paper_2505_11254_gb300 import binding
 from paper_2505_11254_gb300.inputs import (LLAMA8B_N1M, LLAMA8B_N131K, LLAMA8B_N32K, SWEEP_B4_N64K, SWEEP_GAMMAS,
-                                           SWEEP_WINDOWS, generate, to_bits)
+                                           SWEEP_WINDOWS, TINY_N2048, generate, to_bits)
 from gpu_helpers import MAX_ABS, MEAN_ABS
 
 pytestmark = pytest.mark.gpu
@@ -100,6 +101,18 @@ def _prefill(w, q, k, v):
     out = binding.delta_attn_prefill(q, k, v, w.n_sink, w.window, w.gamma, workspace=ws)
     assert binding.check() == binding.DA_OK
     return out
+
+
+def test_tiny_all_elements():
+    """The small configuration (B=1, 4 heads, d=64, N=2048, window 256,
+    gamma 16): every element of the output."""
+    w = TINY_N2048
+    q, k, v = generate(w, device="cuda")
+    out = _prefill(w, q, k, v)
+    ref = oracle.delta_attn(to_bits(q), to_bits(k), to_bits(v), w.n_sink, w.window, w.gamma)["A"]
+    stats = {}
+    _assert_set(w, "all", out.double().cpu().numpy(), ref, stats)
+    _record({"workload": w.name, "window": w.window, "gamma": w.gamma, "pairs": "all", "sets": stats})
 
 
 def test_llama8b_n32k():

@@ -1,5 +1,6 @@
 // Host-side check of the tile geometry in tiles.cuh (compiled as plain C++ by
-// tests/test_tile_geometry.py): for every work item of many shapes and all
+// tests/test_tile_geometry.py): the visibility words the kernels mask scores
+// with match the key sets bit by bit; for every work item of many shapes and all
 // three modes, unmasked_tiles() must select exactly the tiles for which
 // tile_needs_mask() is false, and tile_needs_mask() must be true wherever a
 // (row, key) pair of the tile is not visible (checked pair by pair against
@@ -228,8 +229,29 @@ static int check_shape(int B, int Hq, int Hkv, long long N, long long win, int n
   return bad;
 }
 
+// visible_bits() against the key-set definition, bit by bit: window and
+// causal range [lo, hi] (empty when hi < lo) and sinks c < se.
+static int check_visible_bits() {
+  int bad = 0;
+  const int ses[] = {0, 1, 3, 4, 31, 32, 33, 64, 100, 127, 128};
+  for (int lo = 0; lo <= BN + 1; ++lo)
+    for (int hi = -1; hi < BN; ++hi)
+      for (int se : ses)
+        for (int c0 = 0; c0 < BN; c0 += 32) {
+          const uint32_t v = visible_bits(lo, hi, se, c0);
+          for (int c = c0; c < c0 + 32; ++c) {
+            const bool want = (lo <= c && c <= hi) || c < se;
+            if (((v >> (c - c0)) & 1u) != (want ? 1u : 0u)) {
+              if (bad < 5) std::printf("visible_bits(%d, %d, %d, %d): key %d\n", lo, hi, se, c0, c);
+              ++bad;
+            }
+          }
+        }
+  return bad;
+}
+
 int main() {
-  int bad = 0, cases = 0;
+  int bad = check_visible_bits(), cases = 0;
   const long long Ns[] = {1, 100, 128, 129, 1000, 4097, 20000};
   const long long windows[] = {1, 7, 64, 128, 129, 300, 2048, 100000};
   const int sinks[] = {0, 1, 4, 130, 300};
