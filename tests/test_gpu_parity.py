@@ -35,6 +35,10 @@ CASES = [
     (1, 16, 1, 400, 128, 4, 64, 16),      # GQA 16: 16 heads x 8 samples per dense tile
     (1, 6, 2, 350, 64, 3, 50, 8),         # GQA 3 (not a power of two): one head per dense tile
     (1, 4, 4, 520, 64, 4, 64, 4),         # gamma 4 at d = 64: fused in the tile
+    (1, 4, 2, 1200, 128, 16, 200, 16),    # 16 sinks: the narrow sink tile, every key of it visible
+    (1, 4, 2, 1200, 128, 17, 200, 16),    # 17 sinks: the full-width sink tile
+    (1, 2, 1, 900, 64, 15, 128, 32),      # narrow sink tile at d = 64
+    (1, 2, 2, 1100, 128, 1, 300, 64),     # one sink key
 ]
 
 

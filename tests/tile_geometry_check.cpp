@@ -12,6 +12,7 @@
 #define __host__
 #define __device__
 #define __forceinline__ inline
+#include <algorithm>
 #include <cstdio>
 #include <cstdlib>
 #include <initializer_list>
@@ -55,6 +56,18 @@ static int check(const Params& p, long long items) {
           ++bad;
         }
         h = 1;
+      }
+    }
+    {  // the visited tiles are the sink tiles and the band [kt_lo, kt_hi], each once
+      std::vector<long long> seen;
+      for (int j = 0; j < w.T; ++j) seen.push_back(tile_index(w, j));
+      std::vector<long long> want;
+      for (long long kt = 0; kt < w.n_sink_tiles; ++kt) want.push_back(kt);
+      for (long long kt = w.kt_lo; kt <= w.kt_hi; ++kt) want.push_back(kt);
+      std::sort(seen.begin(), seen.end());
+      if (seen != want || w.n_sink_tiles > w.kt_lo) {
+        if (bad < 5) std::printf("mode %d item %lld: visited tiles are not the sink tiles and the band\n", MODE, it);
+        ++bad;
       }
     }
     for (int j = 0; j < w.T; ++j) {
