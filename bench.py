@@ -33,7 +33,8 @@ process per GPU (torchrun), no collective on the data path; barrier + max over
 ranks around each timed loop.  ``--shard replicas`` (default) runs one
 independent sequence per rank (weak scaling); ``--shard heads`` splits one
 prefill by (batch, KV head) pairs (strong scaling), ``--gather`` then times an
-all-gather of O.
+all-gather of O; ``--shard context`` splits one prefill by rows, each step
+all-gathering the K and V row shards (strong scaling).
 """
 import argparse
 import hashlib
@@ -77,9 +78,9 @@ def parse_args():
     ap.add_argument("--tail", type=int, default=1024, help="dense tail rows of the variant timings")
     ap.add_argument("--no-workloads", action="store_true",
                     help="skip the records of the other configurations (32K, 1M, the B=4 sweep)")
-    ap.add_argument("--shard", choices=["replicas", "heads"], default="replicas",
-                    help="N GPUs: independent sequences (weak scaling) or one prefill split by (batch, KV head) "
-                         "pairs (strong scaling)")
+    ap.add_argument("--shard", choices=["replicas", "heads", "context"], default="replicas",
+                    help="N GPUs: independent sequences (weak scaling), or one prefill split by (batch, KV head) "
+                         "pairs or by rows (strong scaling)")
     ap.add_argument("--gather", action="store_true", help="with --shard heads: time an all-gather of O afterwards")
     return ap.parse_args()
 
@@ -591,6 +592,70 @@ def time_workloads(args, dev, rep, peaks, peak_src):
     return res
 
 
+def run_context(args, w, rep):
+    """One prefill split by rows over the ranks (context parallelism): a step
+    is the all-gather of the K and V row shards and delta_attn_prefill_rows on
+    this rank's rows; barrier and max over ranks around the timed loop."""
+    from paper_2505_11254_gb300 import binding
+    from paper_2505_11254_gb300.replicas import context_shard, gather_kv
+    world, rank, local = rep.world, rep.rank, rep.local
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    q_all, k_all, v_all = generate(w, device=dev)
+    r0, r1 = context_shard(w.N, w.gamma, rank, world)
+    if r1 <= r0:
+        raise RuntimeError("rank %d has no rows: use at most %d GPUs" % (rank, -(-w.N // 128)))
+    q = q_all[:, :, r0:r1].contiguous()
+    k_own, v_own = k_all[:, :, r0:r1].contiguous(), v_all[:, :, r0:r1].contiguous()
+    del q_all, k_all, v_all
+    ws = binding.alloc_workspace(binding.workspace_size_rows(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window,
+                                                             w.gamma, r0, r1 - r0), dev)
+    out = torch.empty_like(q)
+    nk = int(binding.plan_info(w.B, w.Hq, w.Hkv, w.N, w.d, w.n_sink, w.window, w.gamma)["kernels"])
+
+    def step():
+        k, v = gather_kv(k_own, v_own, w.N, w.gamma, world) if world > 1 else (k_own, v_own)
+        binding.delta_attn_prefill_rows(q, k, v, w.n_sink, w.window, w.gamma, r0, out=out, workspace=ws)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if binding.check() != binding.DA_OK:
+        raise RuntimeError("device status after warm-up")
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.25)
+    clocks.mark_start()
+    rep.barrier()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(args.steps):
+        step()
+    t1.record()
+    torch.cuda.synchronize()
+    rep.barrier()
+    clocks.mark_end()
+    clock_info = clocks.stop()
+    if binding.check() != binding.DA_OK:
+        raise RuntimeError("device status after the timed loop")
+    ms_per_step = rep.max(t0.elapsed_time(t1)) / args.steps
+    peaks, _ = load_peaks()
+    peak = float(peaks.get("bf16_tflops", PEAKS_FALLBACK["bf16_tflops"]))
+    useful = flops.useful_flops(w.B, w.Hq, w.N, w.d, w.n_sink, w.window, w.gamma) / (ms_per_step / 1e3) / 1e12
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": w.B * w.N / (ms_per_step / 1e3), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+            "scaling": "strong", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic: seeded N(0,1) Q,K,V, RoPE base 500000 on Q,K, sink keys x%g; no dataset"
+                    % w.sink_scale,
+            "config": dict(config_of(w, world), parallelism="context shards: one prefill split by rows over %d GPUs"
+                           " (all-gather of the K, V row shards each step)" % world),
+            "useful_tflops": useful, "pct_of_bf16_peak": 100 * useful / peak, "rows": [r0, r1],
+            "gpu_launches": nk * args.steps, "clocks": clock_info}), flush=True)
+
+
 def run_ours(args, w, rep):
     from paper_2505_11254_gb300 import binding
     from paper_2505_11254_gb300.replicas import head_shard, shard_views, gather_shards
@@ -711,6 +776,8 @@ def main():
     try:
         if args.impl == "reference":
             run_reference(args, w, rep)
+        elif args.shard == "context":
+            run_context(args, w, rep)
         else:
             run_ours(args, w, rep)
     finally:

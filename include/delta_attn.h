@@ -240,6 +240,27 @@ int delta_attn_prefill_rope(const void* Q, void* K, const void* V, void* O, int 
                             int n_sink, int64_t window, int gamma, const float* table, int64_t table_rows,
                             void* workspace, size_t ws_bytes, void* stream);
 
+/* Rows row_begin .. row_begin + n_rows - 1 of delta_attn_prefill() over a
+ * sequence of N_kv tokens: one rank's share of a sequence split by rows
+ * (context parallelism).  Alg. 1 and Eq. 6 evaluate each row from its own
+ * query and the keys up to it, so the rows of a range need the whole Q and O
+ * of the range only, and K, V up to its last row (the sink keys, the window
+ * before the first row and, for the sampled rows' dense attention, every
+ * earlier key).
+ *   Q, O: [B, Hq, n_rows, d] bf16, row i of the sequence at index i - row_begin;
+ *   K, V: [B, Hkv, N_kv, d] bf16, rows from 0 (rows past row_begin + n_rows are
+ *         not read); row_begin a multiple of 128 and of gamma (the range starts
+ *         a row tile and a sample group), n_rows >= 1, row_begin + n_rows <= N_kv.
+ * The result rows equal those of the whole-sequence call up to the order of
+ * the dense rows' split-K merge.  workspace as delta_attn_prefill(), sized by
+ * delta_attn_workspace_size_rows().  Returns a da_status; asynchronous on
+ * `stream`. */
+int delta_attn_workspace_size_rows(int B, int Hq, int Hkv, int64_t N_kv, int d, int n_sink, int64_t window,
+                                   int gamma, int64_t row_begin, int64_t n_rows, size_t* bytes);
+int delta_attn_prefill_rows(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv,
+                            int64_t N_kv, int d, int n_sink, int64_t window, int gamma, int64_t row_begin,
+                            int64_t n_rows, void* workspace, size_t ws_bytes, void* stream);
+
 /* Workspace bytes delta_attn_prefill_host() needs: two device staging buffers
  * of one (batch, KV head) chunk (its G query heads of Q and O, one K and V
  * head) and the workspace of a chunk's prefill.  Returns a da_status. */

@@ -53,6 +53,8 @@ _SIGNATURES = {
     "delta_attn_rope_table": ([_i64, _i, ctypes.c_double, _p, _p], _i),
     "delta_attn_rope_apply": ([_p, _i, _i, _i64, _i, _i64, _p, _i64, _p], _i),
     "delta_attn_prefill_rope": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _i64, _p, _sz, _p], _i),
+    "delta_attn_workspace_size_rows": ([_i, _i, _i, _i64, _i, _i, _i64, _i, _i64, _i64, ctypes.POINTER(_sz)], _i),
+    "delta_attn_prefill_rows": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _i64, _i64, _p, _sz, _p], _i),
     "delta_attn_host_workspace_size": ([_i, _i, _i, _i64, _i, _i, _i64, _i, ctypes.POINTER(_sz)], _i),
     "delta_attn_prefill_host": ([_p, _p, _p, _p, _i, _i, _i, _i64, _i, _i, _i64, _i, _p, _sz, _p], _i),
     "delta_attn_check": ([_p], _i),
@@ -141,6 +143,34 @@ def strided_dense_workspace_size(B, Hq, Hkv, N, d, gamma) -> int:
     _check(load().strided_dense_workspace_size(B, Hq, Hkv, N, d, gamma, ctypes.byref(out)),
            "strided_dense_workspace_size")
     return out.value
+
+
+def workspace_size_rows(B, Hq, Hkv, N_kv, d, n_sink, window, gamma, row_begin, n_rows) -> int:
+    out = _sz(0)
+    _check(load().delta_attn_workspace_size_rows(B, Hq, Hkv, N_kv, d, n_sink, window, gamma, row_begin, n_rows,
+                                                 ctypes.byref(out)), "delta_attn_workspace_size_rows")
+    return out.value
+
+
+def delta_attn_prefill_rows(q_rows, k, v, n_sink, window, gamma, row_begin, out=None, workspace=None, stream=None):
+    """Rows row_begin .. row_begin + n_rows - 1 of the prefill of a sequence
+    of N_kv tokens (one rank's share under context parallelism): ``q_rows``
+    [B,Hq,n_rows,d] holds those rows of Q, ``k``/``v`` [B,Hkv,N_kv,d] the keys
+    and values from row 0.  Returns bf16 [B,Hq,n_rows,d]."""
+    for name, t in (("q_rows", q_rows), ("k", k), ("v", v)):
+        if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous() or t.dim() != 4:
+            raise ValueError("%s must be a contiguous 4-D bf16 CUDA tensor" % name)
+    B, Hq, n_rows, d = q_rows.shape
+    if k.shape != v.shape or k.shape[0] != B or k.shape[3] != d:
+        raise ValueError("q_rows [B,Hq,n_rows,d], k/v [B,Hkv,N_kv,d]")
+    Hkv, N_kv = k.shape[1], k.shape[2]
+    if out is None:
+        out = torch.empty_like(q_rows)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(load().delta_attn_prefill_rows(_dptr(q_rows), _dptr(k), _dptr(v), _dptr(out), B, Hq, Hkv, N_kv, d, n_sink,
+                                          window, gamma, row_begin, n_rows, _dptr(workspace), ws_bytes,
+                                          _stream(stream)), "delta_attn_prefill_rows")
+    return out
 
 
 def alloc_workspace(nbytes, device):

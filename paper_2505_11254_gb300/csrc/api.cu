@@ -96,8 +96,10 @@ struct Plan {
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
+// N: the end of the rows computed; q_row0: their first row (a row-range call
+// computes rows [q_row0, N) of a longer sequence; 0 for a whole sequence).
 Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t window, int gamma, int sms,
-               int64_t tail = 0, bool smooth = false) {
+               int64_t tail = 0, bool smooth = false, int64_t q_row0 = 0) {
   Plan pl;
   Params& p = pl.p;
   p = Params{};
@@ -109,13 +111,16 @@ Plan make_plan(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, int64_t win
   p.n_sink = n_sink;
   p.window = window;
   p.gamma = gamma;
-  p.n_s = cdiv(N, gamma);
+  p.q_row0 = q_row0;
+  p.o_rows = N - q_row0;
+  p.row0 = q_row0;
+  p.n_s = cdiv(N - q_row0, gamma);
   p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
   packing(p.G, &p.Hp, &p.R);
   p.groups_per_b = Hq / p.Hp;
   // Rows of the dense tail are recomputed densely afterwards, so the sparse
   // pass stops at the q-tile holding row N - tail - 1.
-  p.qtiles = cdiv(N - tail, BM);
+  p.qtiles = cdiv(N - tail - q_row0, BM);
   plan_split_k(p, sms, d);
 
   pl.grid_sparse = (long long)B * Hq * p.qtiles;
@@ -196,20 +201,24 @@ struct Maps {
 };
 
 // Sampled rows row0 + k * gamma of every (b, head): Hp heads x R samples a box.
+// Q holds rows q_row0 .. N - 1 of every (b, head); sample k is row row0 + k gamma.
 bool make_sample_map(CUtensorMap* m, const void* Q, const Params& p, int d) {
   const long long row_bytes = (long long)d * 2;
-  const uint8_t* base = static_cast<const uint8_t*>(Q) + p.row0 * row_bytes;
-  return make_map(m, base, d, p.n_s, row_bytes * p.gamma, (long long)p.B * p.Hq, p.N * row_bytes, p.R, p.Hp);
+  const uint8_t* base = static_cast<const uint8_t*>(Q) + (p.row0 - p.q_row0) * row_bytes;
+  return make_map(m, base, d, p.n_s, row_bytes * p.gamma, (long long)p.B * p.Hq, (p.N - p.q_row0) * row_bytes, p.R,
+                  p.Hp);
 }
 
+// n_kv: rows K and V hold per (b, KV head), at least p.N.
 bool make_maps(Maps* m, const void* Q, const void* K, const void* V, const Params& p, int d, bool need_rows,
-               bool need_samples) {
+               bool need_samples, long long n_kv) {
   const long long row_bytes = (long long)d * 2;
-  if (need_rows && !make_map(&m->q, Q, d, p.N, row_bytes, (long long)p.B * p.Hq, p.N * row_bytes, BM, 1))
+  const long long q_rows = p.N - p.q_row0;
+  if (need_rows && !make_map(&m->q, Q, d, q_rows, row_bytes, (long long)p.B * p.Hq, q_rows * row_bytes, BM, 1))
     return false;
   if (need_samples && !make_sample_map(&m->qs, Q, p, d)) return false;
-  if (!make_map(&m->k, K, d, p.N, row_bytes, (long long)p.B * p.Hkv, p.N * row_bytes, BN, 1)) return false;
-  if (!make_map(&m->v, V, d, p.N, row_bytes, (long long)p.B * p.Hkv, p.N * row_bytes, BN, 1)) return false;
+  if (!make_map(&m->k, K, d, n_kv, row_bytes, (long long)p.B * p.Hkv, n_kv * row_bytes, BN, 1)) return false;
+  if (!make_map(&m->v, V, d, n_kv, row_bytes, (long long)p.B * p.Hkv, n_kv * row_bytes, BN, 1)) return false;
   return true;
 }
 
@@ -218,6 +227,16 @@ cudaError_t launch(int d, const CUtensorMap& q, const CUtensorMap& k, const CUte
                    long long grid, cudaStream_t s) {
   if (d == 64) return launch_attn<64, MODE, EPI>(q, k, v, p, grid, s);
   return launch_attn<128, MODE, EPI>(q, k, v, p, grid, s);
+}
+
+// The sink + window pass of a row-range call: the ROWS instance when the range
+// starts after row 0.
+template <int EPI>
+cudaError_t launch_sparse(int d, const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v, const Params& p,
+                          long long grid, cudaStream_t s) {
+  if (p.q_row0 == 0) return launch<MODE_SPARSE, EPI>(d, q, k, v, p, grid, s);
+  if (d == 64) return launch_attn<64, MODE_SPARSE, EPI, true>(q, k, v, p, grid, s);
+  return launch_attn<128, MODE_SPARSE, EPI, true>(q, k, v, p, grid, s);
 }
 
 class ScopedWorkspace {
@@ -389,10 +408,22 @@ int delta_attn_plan_info(int B, int Hq, int Hkv, int64_t N, int d, int n_sink, i
 // rope: a (cos, sin) table [>= N][d/2][2] when Q and K come unrotated; K is
 // then rotated in place before the first kernel and every Q tile on its way
 // into tensor memory.
+// A row range of a longer sequence (delta_attn_prefill_rows): rows
+// [q_row0, N) with K and V of n_kv rows; {0, 0} for a whole sequence.
+struct RowRange {
+  int64_t q_row0 = 0, n_kv = 0;
+};
+
+static int check_rows(int64_t N_kv, int gamma, int64_t row_begin, int64_t n_rows) {
+  if (row_begin < 0 || n_rows < 1 || gamma < 1 || row_begin > N_kv - n_rows) return DA_ERR_INVALID_ARG;
+  if (row_begin % BM != 0 || row_begin % gamma != 0) return DA_ERR_INVALID_ARG;
+  return DA_OK;
+}
+
 static int prefill_impl(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv, int64_t N,
                         int d, int n_sink, int64_t window, int gamma, int mode, int64_t tail, const SmoothArgs& sm,
                         void* workspace, size_t ws_bytes, void* stream, void* const* events, int n_events,
-                        const float* rope = nullptr) {
+                        const float* rope = nullptr, RowRange rr = RowRange{}) {
   if (!Q || !K || !V || !O) return DA_ERR_INVALID_ARG;
   int rc = check_shape(B, Hq, Hkv, N, d, n_sink, window, gamma);
   if (rc) return rc;
@@ -404,7 +435,14 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   int sms = 0;
   if ((rc = check_device(&sms))) return rc;
   const bool smooth = sm.kind != DA_SMOOTH_NONE;
-  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms, tail, smooth);
+  Plan pl = make_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, sms, tail, smooth, rr.q_row0);
+  // A row range: the passes that index O by absolute row, and the per-sample
+  // buffers by absolute sample, get base pointers moved back by the range's
+  // first row (sample), so the kernels' indexing is that of a whole sequence.
+  // Only rows and samples inside the range are ever addressed through them.
+  const long long s_off = rr.q_row0 / gamma;
+  void* const O_abs = static_cast<uint8_t*>(O) - rr.q_row0 * (long long)d * 2;
+  auto abs_samples = [&](float* f) { return f - s_off * d; };
   const int n_kernels = prefill_kernels(pl, gamma, mode);
   if (n_events != 0 && (events == nullptr || n_events != n_kernels + 1)) return DA_ERR_INVALID_ARG;
   if (workspace != nullptr && ws_bytes < pl.total) return DA_ERR_WORKSPACE;
@@ -412,7 +450,8 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   Params p = pl.p;
   if ((rc = status_ptr(&p.err))) return rc;
   Maps m;
-  if (!make_maps(&m, Q, K, V, p, d, gamma >= 2 || smooth, true)) return DA_ERR_INVALID_ARG;
+  if (!make_maps(&m, Q, K, V, p, d, gamma >= 2 || smooth, true, rr.n_kv > 0 ? rr.n_kv : N))
+    return DA_ERR_INVALID_ARG;
   CUtensorMap q_tail;
   if (pl.tail > 0 && !make_sample_map(&q_tail, Q, pl.pt, d)) return DA_ERR_INVALID_ARG;
 
@@ -472,8 +511,8 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
     e = launch_delta_smooth(delta, basis, coef, (long long)B * Hq, p.n_s, d, gamma, pl.n_coef, sm.kind, sm.c1, sm.c2,
                             sm.c3, s);
     if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
-    p.out_bf16 = O;
-    p.smooth_basis = basis;
+    p.out_bf16 = O_abs;
+    p.smooth_basis = basis - s_off * kSmoothJ * d;  // kSmoothJ vectors per sample
     p.smooth_coef = coef;
     e = launch<MODE_SPARSE, EPI_FUSED_SMOOTH>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
     if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
@@ -481,14 +520,14 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   }
   if (gamma == 1) {
     // Every row is a sampled row: the output is dense causal attention.
-    p.out_bf16 = O;
+    p.out_bf16 = O_abs;
     e = launch<MODE_STRIDED_DENSE, EPI_DENSE_BF16>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
     return (e == cudaSuccess && mark()) ? DA_OK : DA_ERR_CUDA;
   }
   if (mode == DA_MODE_RECOMPUTE) {
     // Eq. 5: sparse rows everywhere, then the sampled rows overwritten by
     // their dense rows; no correction reaches the other rows.
-    p.out_bf16 = O;
+    p.out_bf16 = O_abs;
     e = launch<MODE_SPARSE, EPI_BF16>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
     if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
     e = launch<MODE_STRIDED_DENSE, EPI_DENSE_BF16>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
@@ -500,18 +539,20 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   e = launch<MODE_STRIDED_DENSE, EPI_DENSE_F32>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
   if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
   p.d_out = nullptr;
-  p.d_in = dbuf;
-  p.out_bf16 = O;
+  p.out_bf16 = O_abs;
   if (pl.fused_intile) {
-    e = launch<MODE_SPARSE, EPI_FUSED_INTILE>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+    p.d_in = abs_samples(dbuf);
+    e = launch_sparse<EPI_FUSED_INTILE>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
   } else {
     float* delta = reinterpret_cast<float*>(base + pl.off_delta);
+    p.d_in = dbuf;  // the strided sparse pass indexes its own samples
     p.delta_out = delta;
     e = launch<MODE_STRIDED_SPARSE, EPI_DELTA_BUILD>(d, m.qs, m.k, m.v, p, pl.grid_ssparse, s);
     if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
     p.delta_out = nullptr;
-    p.delta_in = delta;
-    e = launch<MODE_SPARSE, EPI_FUSED_DELTA>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+    p.d_in = abs_samples(dbuf);
+    p.delta_in = abs_samples(delta);
+    e = launch_sparse<EPI_FUSED_DELTA>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
   }
   if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
   return run_tail();
@@ -565,7 +606,7 @@ int sparse_window_attn(const void* Q, const void* K, const void* V, void* O_spar
   Params p = pl.p;
   if ((rc = status_ptr(&p.err))) return rc;
   Maps m;
-  if (!make_maps(&m, Q, K, V, p, d, true, false)) return DA_ERR_INVALID_ARG;
+  if (!make_maps(&m, Q, K, V, p, d, true, false, N)) return DA_ERR_INVALID_ARG;
   p.out_bf16 = O_sparse;
   p.s_sampled = S_sampled;
   cudaError_t e = launch<MODE_SPARSE, EPI_BF16>(d, m.q, m.k, m.v, p, pl.grid_sparse, static_cast<cudaStream_t>(stream));
@@ -587,7 +628,7 @@ int strided_dense_attn(const void* Q, const void* K, const void* V, float* D_sam
   Params p = pl.p;
   if ((rc = status_ptr(&p.err))) return rc;
   Maps m;
-  if (!make_maps(&m, Q, K, V, p, d, false, true)) return DA_ERR_INVALID_ARG;
+  if (!make_maps(&m, Q, K, V, p, d, false, true, N)) return DA_ERR_INVALID_ARG;
   ScopedWorkspace ws(workspace, pl.dense_total, s);
   if (ws.failed()) return DA_ERR_CUDA;
   p.partials = reinterpret_cast<float*>(ws.get() + pl.dense_part);
@@ -687,6 +728,28 @@ int delta_attn_prefill_rope(const void* Q, void* K, const void* V, void* O, int 
   if (!table || table_rows < N) return DA_ERR_INVALID_ARG;
   return prefill_impl(Q, K, V, O, B, Hq, Hkv, N, d, n_sink, window, gamma, DA_MODE_DELTA, 0, SmoothArgs{},
                       workspace, ws_bytes, stream, nullptr, 0, table);
+}
+
+int delta_attn_workspace_size_rows(int B, int Hq, int Hkv, int64_t N_kv, int d, int n_sink, int64_t window,
+                                   int gamma, int64_t row_begin, int64_t n_rows, size_t* bytes) {
+  if (!bytes) return DA_ERR_INVALID_ARG;
+  int rc = check_shape(B, Hq, Hkv, N_kv, d, n_sink, window, gamma);
+  if (rc) return rc;
+  if ((rc = check_rows(N_kv, gamma, row_begin, n_rows))) return rc;
+  int sms = 0;
+  if ((rc = check_device(&sms))) return rc;
+  *bytes = make_plan(B, Hq, Hkv, row_begin + n_rows, d, n_sink, window, gamma, sms, 0, false, row_begin).total;
+  return DA_OK;
+}
+
+int delta_attn_prefill_rows(const void* Q, const void* K, const void* V, void* O, int B, int Hq, int Hkv,
+                            int64_t N_kv, int d, int n_sink, int64_t window, int gamma, int64_t row_begin,
+                            int64_t n_rows, void* workspace, size_t ws_bytes, void* stream) {
+  int rc = check_shape(B, Hq, Hkv, N_kv, d, n_sink, window, gamma);
+  if (rc) return rc;
+  if ((rc = check_rows(N_kv, gamma, row_begin, n_rows))) return rc;
+  return prefill_impl(Q, K, V, O, B, Hq, Hkv, row_begin + n_rows, d, n_sink, window, gamma, DA_MODE_DELTA, 0,
+                      SmoothArgs{}, workspace, ws_bytes, stream, nullptr, 0, nullptr, RowRange{row_begin, N_kv});
 }
 
 int delta_attn_check(void* stream) {

@@ -225,7 +225,10 @@ struct ItemReader {
   }
 };
 
-template <int D, int MODE, int EPI>
+// ROWS: the kernel of a row-range call (Params::q_row0 > 0): items start at
+// row q_row0, Q and O hold rows from q_row0.  Whole-sequence launches use
+// ROWS = false.
+template <int D, int MODE, int EPI, bool ROWS = false>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const Params p) {
@@ -300,15 +303,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       int c = 0, nq = 0;
       bool ok = true;
       auto load_q = [&](long long item) {
-        const Work wq = decode_work<MODE>(p, item);
+        const Work wq = decode_work<MODE, ROWS>(p, item);
         // buffer qb held the Q of item nq - NQ: its last QK (or, Q in TMEM, the
         // epilogue's copy) must have read it
         const int qb = nq % C::NQ;
         if (nq >= C::NQ && !wait_bounded(&bars.q_free[qb], ((nq / C::NQ) - 1) & 1, &abort_sh, p.err)) return false;
         mbar_arrive_expect_tx(&bars.q_full[qb], C::Q_BYTES);
         for (int ch = 0; ch < C::CHUNKS; ++ch)
-          tma_load_3d(sQ + qb * C::Q_BYTES + ch * (BM * 128), &tmQ, &bars.q_full[qb], ch * 64, (int)wq.r0,
-                      wq.b * p.Hq + wq.h0);
+          tma_load_3d(sQ + qb * C::Q_BYTES + ch * (BM * 128), &tmQ, &bars.q_full[qb], ch * 64,
+                      (int)(ROWS && MODE == MODE_SPARSE ? wq.r0 - p.q_row0 : wq.r0), wq.b * p.Hq + wq.h0);
         ++nq;
         return true;
       };
@@ -351,7 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       long long item = claim();
       if (item >= 0) ok = load_q(item);
       while (ok && item >= 0) {
-        const Work w = decode_work<MODE>(p, item);
+        const Work w = decode_work<MODE, ROWS>(p, item);
         const int kz = w.b * p.Hkv + w.g;
         long long nxt = -1;
         for (int j = 0; ok && j < w.T; ++j) {
@@ -388,7 +391,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ItemReader<DYN, false> items{(long long)blockIdx.x};
       int i = 0;
       for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
-        const Work w = decode_work<MODE>(p, item);
+        const Work w = decode_work<MODE, ROWS>(p, item);
         // Q of item i: in TMEM buffer i & 1 (copied by the epilogue), or in smem
         // buffer i % NQ (rotated in place first when RoPE is on)
         const int qb = C::QTMEM ? (i & 1) : i % C::NQ;
@@ -440,7 +443,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ItemReader<DYN, false> items{(long long)blockIdx.x};
       int i = 0;
       for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
-        const Work w = decode_work<MODE>(p, item);
+        const Work w = decode_work<MODE, ROWS>(p, item);
         for (int j = 0; j < w.T; ++j, ++g) {
           const int vs = (int)(g % C::NV);
           const uint32_t vph = (uint32_t)(g / C::NV) & 1;
@@ -474,7 +477,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       ItemReader<DYN, false> items{(long long)blockIdx.x};
       for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh)) {
-        const Work w = decode_work<MODE>(p, item);
+        const Work w = decode_work<MODE, ROWS>(p, item);
         const int kz = w.b * p.Hkv + w.g;
         for (int j = 0; ok && j < w.T; ++j) {
           const int s = c % C::NV;
@@ -505,7 +508,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int i = 0;
     ItemReader<DYN, true> items{(long long)blockIdx.x};
     for (long long item = items.next(p, iq, &abort_sh); item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
-      const Work w = decode_work<MODE>(p, item);
+      const Work w = decode_work<MODE, ROWS>(p, item);
       long long row, sample;
       int head;
       lane_row<MODE>(p, w, t, row, sample, head);
@@ -657,7 +660,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             r[ch * 32 + pc * 4 + 3] = v.w;
           }
         if (p.rope != nullptr) {
-          const Work wq = decode_work<MODE>(p, qitem);
+          const Work wq = decode_work<MODE, ROWS>(p, qitem);
           long long qrow, qsample;
           int qhead;
           if (lane_row<MODE>(p, wq, e, qrow, qsample, qhead)) {
@@ -695,7 +698,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (p.rope == nullptr) return;
       ok = ok && __all_sync(kFull, wait_sleepy(&bars.q_full[buf], (nq / C::NQ) & 1, &abort_sh, p.err));
       ++nq;
-      const Work wq = decode_work<MODE>(p, qitem);
+      const Work wq = decode_work<MODE, ROWS>(p, qitem);
       long long qrow, qsample;
       int qhead;
       if (ok && lane_row<MODE>(p, wq, e, qrow, qsample, qhead)) {
@@ -736,7 +739,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     long long item = items.next(p, iq, &abort_sh);
     if (item >= 0) rotate_q(0, item);
     for (int i = 0; item >= 0; ++i) {
-      const Work w = decode_work<MODE>(p, item);
+      const Work w = decode_work<MODE, ROWS>(p, item);
       const long long nxt = items.next(p, iq, &abort_sh);
       if (nxt >= 0) rotate_q(C::QTMEM ? ((i + 1) & 1) : (i + 1) % C::NQ, nxt);
       long long row, sample;
@@ -756,6 +759,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const long long bh = (long long)w.b * p.Hq + head;
       const float inv_l = (l_row > 0.f) ? 1.f / l_row : 0.f;
 
+
       if (EPI == EPI_BF16 || EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA || EPI == EPI_DELTA_BUILD ||
           EPI == EPI_FUSED_SMOOTH) {
 #pragma unroll
@@ -772,7 +776,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           named_bar_sync(2, 128);
         }
         if (ok && row_ok) {
-          __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out_bf16) + (bh * p.N + row) * D;
+          __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out_bf16) + (bh * (ROWS ? p.o_rows : p.N) + row) * D;
 #pragma unroll
           for (int q = 0; q < D / 32; ++q) {
             float* v = o + q * 32;
@@ -824,7 +828,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (EPI == EPI_DENSE_F32)
             store_f32x32(p.d_out + (bh * p.n_s + sample) * D + q * 32, v);
           else
-            store_bf16x32(reinterpret_cast<__nv_bfloat16*>(p.out_bf16) + (bh * p.N + row) * D + q * 32, v);
+            store_bf16x32(reinterpret_cast<__nv_bfloat16*>(p.out_bf16) + (bh * p.o_rows + row) * D + q * 32, v);
         };
         if (w.n_chunks == 1) {
           if (ok && row_ok) {

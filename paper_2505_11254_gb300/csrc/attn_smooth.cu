@@ -4,10 +4,10 @@
 #include "launch_impl.cuh"
 
 namespace da {
-template cudaError_t launch_attn<64, MODE_SPARSE, EPI_FUSED_SMOOTH>(const CUtensorMap&, const CUtensorMap&,
+template cudaError_t launch_attn<64, MODE_SPARSE, EPI_FUSED_SMOOTH, false>(const CUtensorMap&, const CUtensorMap&,
                                                                     const CUtensorMap&, const Params&, long long,
                                                                     cudaStream_t);
-template cudaError_t launch_attn<128, MODE_SPARSE, EPI_FUSED_SMOOTH>(const CUtensorMap&, const CUtensorMap&,
+template cudaError_t launch_attn<128, MODE_SPARSE, EPI_FUSED_SMOOTH, false>(const CUtensorMap&, const CUtensorMap&,
                                                                      const CUtensorMap&, const Params&, long long,
                                                                      cudaStream_t);
 }  // namespace da

@@ -3,10 +3,10 @@
 #include "launch_impl.cuh"
 
 namespace da {
-template cudaError_t launch_attn<64, MODE_STRIDED_SPARSE, EPI_DELTA_BUILD>(const CUtensorMap&, const CUtensorMap&,
+template cudaError_t launch_attn<64, MODE_STRIDED_SPARSE, EPI_DELTA_BUILD, false>(const CUtensorMap&, const CUtensorMap&,
                                                                            const CUtensorMap&, const Params&,
                                                                            long long, cudaStream_t);
-template cudaError_t launch_attn<128, MODE_STRIDED_SPARSE, EPI_DELTA_BUILD>(const CUtensorMap&,
+template cudaError_t launch_attn<128, MODE_STRIDED_SPARSE, EPI_DELTA_BUILD, false>(const CUtensorMap&,
                                                                             const CUtensorMap&,
                                                                             const CUtensorMap&, const Params&,
                                                                             long long, cudaStream_t);

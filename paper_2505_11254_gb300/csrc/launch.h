@@ -9,7 +9,8 @@
 
 namespace da {
 
-template <int D, int MODE, int EPI>
+// ROWS: the instance for row-range calls (rows from Params::q_row0 > 0).
+template <int D, int MODE, int EPI, bool ROWS = false>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
                         long long n_items, cudaStream_t s);
 

@@ -7,10 +7,10 @@ namespace da {
 
 // Persistent launch: min(items, SMs) CTAs, each walking items with a stride
 // of the grid size.
-template <int D, int MODE, int EPI>
+template <int D, int MODE, int EPI, bool ROWS>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
                         long long n_items, cudaStream_t s) {
-  auto kfn = attn_kernel<D, MODE, EPI>;
+  auto kfn = attn_kernel<D, MODE, EPI, ROWS>;
   cudaError_t e = cudaFuncSetAttribute(kfn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg<D, MODE>::SMEM);
   if (e != cudaSuccess) return e;
   if (n_items <= 0) return cudaSuccess;

@@ -57,8 +57,16 @@ struct Params {
   int n_sink;
   long long window;
   int gamma;
-  long long n_s;           // number of sampled rows ceil(N / gamma)
-  long long row0;          // row of sample 0: 0, or N - t for the dense tail block of t rows
+  long long n_s;           // sampled rows the call computes (ceil((N - q_row0) / gamma); the tail's rows)
+  long long row0;          // row of sample 0: q_row0, or N - t for the dense tail block of t rows
+  // Rows computed: [q_row0, N).  Q holds exactly these rows (row i at index
+  // i - q_row0); K and V hold rows from 0.  A whole-sequence call has
+  // q_row0 = 0; a row-range call (one rank's share of a sequence) has q_row0
+  // a multiple of BM and of gamma, and the host passes the output and the
+  // per-sample buffers the sink + window pass reads by absolute row or sample
+  // as base pointers moved back by q_row0 rows (q_row0 / gamma samples).
+  long long q_row0;
+  long long o_rows;        // rows per (b, head) of the output buffer (its row stride)
   float scale_log2;        // log2(e) / sqrt(d)
   // sampled-row packing: Hp heads x R samples per tile (Hp * R == BM)
   int Hp, R;
@@ -233,7 +241,7 @@ __host__ __device__ inline Work decode_strided_dense(const Params& p, long long 
 
 // Contiguous rows: CTA order is (kv-head group member fastest, q-tile, kv-head,
 // batch) so the G query heads that share K/V run side by side.
-__host__ __device__ inline Work decode_sparse(const Params& p, long long lin) {
+__host__ __device__ inline Work decode_sparse(const Params& p, long long lin, long long row_off) {
   Work w;
   int hl;
   long long qt;
@@ -257,7 +265,7 @@ __host__ __device__ inline Work decode_sparse(const Params& p, long long lin) {
     w.b = (int)(lin / p.Hkv);
   }
   w.h0 = w.g * p.G + hl;
-  w.r0 = qt * BM;
+  w.r0 = row_off + qt * BM;
   w.r_last = lmin(w.r0 + BM, p.N) - 1;
   long long band_lo = lmax(0, w.r0 - p.window + 1);
   w.kt_lo = band_lo / BN;
@@ -281,7 +289,7 @@ __host__ __device__ inline Work decode_strided_sparse(const Params& p, long long
   w.g = w.h0 / p.G;
   w.r0 = t * p.R;
   w.r_last = lmin(w.r0 + p.R - 1, p.n_s - 1);
-  long long row_first = w.r0 * p.gamma, row_last = w.r_last * p.gamma;
+  long long row_first = p.row0 + w.r0 * p.gamma, row_last = p.row0 + w.r_last * p.gamma;
   w.kt_lo = lmax(0, row_first - p.window + 1) / BN;
   w.kt_hi = row_last / BN;
   w.n_sink_tiles = sink_tiles_before(p.n_sink, row_last, w.kt_lo);
@@ -292,9 +300,11 @@ __host__ __device__ inline Work decode_strided_sparse(const Params& p, long long
   return w;
 }
 
-template <int MODE>
+// ROWS: a row-range call (rows from p.q_row0); whole-sequence kernels are
+// compiled with ROWS = false and start at row 0.
+template <int MODE, bool ROWS = false>
 __host__ __device__ __forceinline__ Work decode_work(const Params& p, long long lin) {
-  if (MODE == MODE_SPARSE) return decode_sparse(p, lin);
+  if (MODE == MODE_SPARSE) return decode_sparse(p, lin, ROWS ? p.q_row0 : 0);
   if (MODE == MODE_STRIDED_DENSE) return decode_strided_dense(p, lin);
   return decode_strided_sparse(p, lin);
 }
@@ -315,7 +325,7 @@ __host__ __device__ __forceinline__ bool tile_needs_mask(const Params& p, const 
   } else if (MODE == MODE_STRIDED_DENSE) {
     return !(k_end <= p.row0 + w.r0 * p.gamma);
   } else {
-    return !(k_end <= w.r0 * p.gamma && k_first > w.r_last * p.gamma - p.window);
+    return !(k_end <= p.row0 + w.r0 * p.gamma && k_first > p.row0 + w.r_last * p.gamma - p.window);
   }
 }
 
@@ -331,9 +341,8 @@ __host__ __device__ __forceinline__ long long floor_div(long long a, long long b
 // is two integer compares.
 template <int MODE>
 __host__ __device__ __forceinline__ void unmasked_tiles(const Params& p, const Work& w, int& j0, int& j1) {
-  const long long rf = (MODE == MODE_SPARSE) ? w.r0
-                       : (MODE == MODE_STRIDED_DENSE) ? p.row0 + w.r0 * p.gamma : w.r0 * p.gamma;
-  const long long rl = (MODE == MODE_SPARSE) ? w.r_last : w.r_last * p.gamma;
+  const long long rf = (MODE == MODE_SPARSE) ? w.r0 : p.row0 + w.r0 * p.gamma;
+  const long long rl = (MODE == MODE_SPARSE) ? w.r_last : p.row0 + w.r_last * p.gamma;
   const long long k_causal = floor_div(rf - (BN - 1), BN);  // last tile all rows see causally
   const long long k_window = (MODE == MODE_STRIDED_DENSE) ? w.kt_lo : floor_div(rl - p.window, BN) + 1;
   const long long lo = lmax(w.kt_lo, k_window), hi = lmin(w.kt_hi, k_causal);

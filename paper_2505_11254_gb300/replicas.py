@@ -6,7 +6,9 @@ groups with their query heads) with no exchange.  Two ways to use N GPUs, one
 process per GPU (launched by torchrun), no collective on the data path:
   * replicas: N independent seeded sequences, one per rank (weak scaling);
   * head shards: one prefill whose (batch, KV head) pairs are split over the
-    ranks (strong scaling), optionally followed by an all-gather of O.
+    ranks (strong scaling), optionally followed by an all-gather of O;
+  * context shards: one prefill split by rows, after an all-gather of the K
+    and V row shards (strong scaling).
 Timing uses a barrier on both sides of the timed loop and the maximum of the
 per-rank times; whole-job throughput is the work of all ranks over that time.
 
@@ -115,3 +117,54 @@ def gather_shards(O_part, B: int, Hq: int, Hkv: int, world: int):
     for (p0, p1), buf in zip(ranges, bufs):
         out[p0:p1].copy_(buf[: p1 - p0])
     return out.reshape(B, Hq, N, d)
+
+
+# ------------------------------------------------------------ context shards
+# One sequence split by rows (context parallelism).  Rank r computes the rows
+# [r0, r1) of every (b, head) with delta_attn_prefill_rows from its rows of Q
+# and the keys and values of rows 0 .. r1 - 1: the sink keys, the window before
+# r0 and, for its sampled rows' dense attention, every earlier key.  The one
+# exchange is an all-gather of the K and V row shards; a range starts on a
+# 128-row tile and a sample group, so its correction needs no other rank's Q.
+
+def context_shard(N: int, gamma: int, rank: int, world: int):
+    """Row range [r0, r1) of rank `rank`: the sequence cut at multiples of
+    lcm(128, gamma) into `world` ranges whose unit counts differ by at most
+    one (a rank may get none when the sequence has fewer units than ranks)."""
+    import math
+    if world < 1 or not 0 <= rank < world:
+        raise ValueError("rank %d outside a world of %d" % (rank, world))
+    unit = math.lcm(128, gamma)
+    n_units = -(-N // unit)
+    u0, u1 = rank * n_units // world, (rank + 1) * n_units // world
+    return min(u0 * unit, N), min(u1 * unit, N)
+
+
+def _gather_rows(part, N: int, gamma: int, world: int):
+    """All-gather of per-rank row ranges [.., r1 - r0, ..] (dim 2) into the
+    whole [.., N, ..] tensor on every rank (padded to the longest range)."""
+    import torch.distributed as dist
+    ranges = [context_shard(N, gamma, r, world) for r in range(world)]
+    width = max(r1 - r0 for r0, r1 in ranges)
+    shape = list(part.shape)
+    shape[2] = width
+    pad = part.new_zeros(shape)
+    pad[:, :, : part.shape[2]].copy_(part)
+    bufs = [torch.empty_like(pad) for _ in range(world)]
+    dist.all_gather(bufs, pad)
+    shape[2] = N
+    out = part.new_empty(shape)
+    for (r0, r1), buf in zip(ranges, bufs):
+        out[:, :, r0:r1].copy_(buf[:, :, : r1 - r0])
+    return out
+
+
+def gather_kv(K_part, V_part, N: int, gamma: int, world: int):
+    """The context-parallel exchange: every rank's rows of K and V gathered
+    into the whole [B, Hkv, N, d] K and V on every rank."""
+    return _gather_rows(K_part, N, gamma, world), _gather_rows(V_part, N, gamma, world)
+
+
+def gather_context(O_part, N: int, gamma: int, world: int):
+    """All-gather of the per-rank output rows into the whole [B, Hq, N, d] O."""
+    return _gather_rows(O_part, N, gamma, world)

@@ -35,7 +35,7 @@ static int check(const Params& p, long long items) {
   const long long per_head = MODE == MODE_SPARSE ? p.N : p.n_s;
   std::vector<unsigned char> held(MODE == MODE_STRIDED_DENSE ? 0 : (size_t)p.B * p.Hq * per_head, 0);
   for (long long it = 0; it < items; ++it) {
-    Work w = decode_work<MODE>(p, it);
+    Work w = p.q_row0 > 0 ? decode_work<MODE, true>(p, it) : decode_work<MODE>(p, it);
     int j0, j1;
     unmasked_tiles<MODE>(p, w, j0, j1);
     for (int t = 0; t < BM; ++t) {  // GQA: every lane's query head reads the item's KV head
@@ -95,9 +95,11 @@ static int check(const Params& p, long long items) {
       }
     }
   }
+  // rows (samples) from the call's first one are each held once; earlier ones never
+  const long long first = MODE == MODE_SPARSE ? p.q_row0 : 0;
   for (size_t i = 0; i < held.size(); ++i)
-    if (!held[i]) {
-      if (bad < 5) std::printf("mode %d: (b, head, row) %zu held by no lane\n", MODE, i);
+    if ((long long)(i % per_head) >= first ? !held[i] : held[i]) {
+      if (bad < 5) std::printf("mode %d: (b, head, row) %zu held %d times\n", MODE, i, (int)held[i]);
       ++bad;
     }
   return bad;
@@ -208,14 +210,16 @@ static const PlanCase kPlans[] = {{152, {kMaxLevelsUsed, kUnitTiles, kMinChunk, 
                                   {152, {kMaxLevelsUsed, 3, 1, 0}},
                                   {1, {kMaxLevels, 1, 1, kLevelPartialBytes}}};
 
-static int check_shape(int B, int Hq, int Hkv, long long N, long long win, int ns, int gm) {
+// q_row0: a row-range call computing rows [q_row0, N) (0: the whole sequence).
+static int check_shape(int B, int Hq, int Hkv, long long N, long long win, int ns, int gm, long long q_row0 = 0) {
   int bad = 0;
   Params p = {};
   p.B = B; p.Hq = Hq; p.Hkv = Hkv; p.G = Hq / Hkv; p.N = N; p.n_sink = ns; p.window = win; p.gamma = gm;
-  p.n_s = (N + gm - 1) / gm;
+  p.q_row0 = q_row0; p.row0 = q_row0; p.o_rows = N - q_row0;
+  p.n_s = (N - q_row0 + gm - 1) / gm;
   packing(p.G, &p.Hp, &p.R);
   p.groups_per_b = p.Hq / p.Hp;
-  p.qtiles = (N + BM - 1) / BM;
+  p.qtiles = (N - q_row0 + BM - 1) / BM;
   plan_split_k(p, 152, 128);
   bad += check<MODE_SPARSE>(p, (long long)p.B * p.Hq * p.qtiles);
   bad += check<MODE_STRIDED_SPARSE>(p, (long long)p.B * p.groups_per_b * p.mtiles);
@@ -284,6 +288,17 @@ int main() {
         for (int ns : {0, 4, 300})
           for (int gm : {1, 3, 16, 64}) {
             bad += check_shape(hk[0], hk[1], hk[2], N, win, ns, gm);
+            ++cases;
+          }
+  // row ranges of a longer sequence (context parallelism): the first row a
+  // multiple of 128 and of gamma
+  for (long long N : {1000LL, 4097LL, 20000LL})
+    for (long long win : {1LL, 300LL, 2048LL})
+      for (int ns : {0, 4, 300})
+        for (int gm : {1, 16, 64, 3, 48})
+          for (long long q_row0 : {128LL * 3, 128LL * 48, 128LL * 96}) {
+            if (q_row0 % gm != 0 || q_row0 >= N) continue;
+            bad += check_shape(1, 4, 2, N, win, ns, gm, q_row0);
             ++cases;
           }
   std::printf("%d shapes, %d mismatches\n", cases, bad);
