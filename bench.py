@@ -448,9 +448,11 @@ def time_prefill(w, q, k, v, steps, warmup, rep, peaks, peak_src, local, min_sec
     repeated back to back (each repeat bracketed by a barrier and a device
     synchronize, the max over ranks taken per repeat) until the timed region
     lasts about `min_seconds` (about 50 clock samples at one per 20 ms).
-    The library records CUDA events between its
-    kernels on the launching stream, which give the per-kernel times.  Returns
-    (record, out) with out holding the last step's result."""
+    A second loop of as many calls, right after, has the library record CUDA
+    events between its kernels on the launching stream: those give the
+    per-kernel times (each kernel then runs alone, without the overlap of a
+    programmatic dependent launch).  Returns (record, out) with out holding
+    the last step's result."""
     from paper_2505_11254_gb300 import binding
     B, Hq, Hkv, N, d = q.shape[0], q.shape[1], k.shape[1], q.shape[2], q.shape[3]
     info = binding.plan_info(B, Hq, Hkv, N, d, w.n_sink, w.window, w.gamma)
@@ -480,7 +482,8 @@ def time_prefill(w, q, k, v, steps, warmup, rep, peaks, peak_src, local, min_sec
     est_ms = rep.max(e0.elapsed_time(e1))
     repeats = max(1, min(max_repeats, int(-(-min_seconds * 1e3 // (steps * est_ms)))))
 
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(steps * repeats)]
+    n_ev = min(steps * repeats, max(steps, 40))
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(n_ev)]
     for row in evs:
         for e in row:
             e.record(stream)  # create the events before the timed region
@@ -499,12 +502,15 @@ def time_prefill(w, q, k, v, steps, warmup, rep, peaks, peak_src, local, min_sec
         t_end = torch.cuda.Event(enable_timing=True)
         t_start.record(stream)
         for s in range(steps):
-            step(evs[r * steps + s])
+            step()
         t_end.record(stream)
         torch.cuda.synchronize()
         rep.barrier()
         loop_ms.append(rep.max(t_start.elapsed_time(t_end)))
     clocks.mark_end()
+    for row in evs:  # per-kernel times
+        step(row)
+    torch.cuda.synchronize()
     clock_info = clocks.stop()
     status = binding.check()
     if status != binding.DA_OK:
