@@ -53,7 +53,7 @@ import torch  # noqa: E402
 
 from paper_2505_11254_gb300 import flops  # noqa: E402
 from paper_2505_11254_gb300.replicas import Replicas  # noqa: E402
-from paper_2505_11254_gb300.inputs import WORKLOADS, LLAMA8B_N131K, generate, to_bits  # noqa: E402
+from paper_2505_11254_gb300.inputs import WORKLOADS, LLAMA8B_N131K, checksums, generate, to_bits  # noqa: E402
 
 METRIC = "Δ-attn prefill tokens/s and useful TFLOP/s (% bf16 tensor peak) at N=131K/1M"
 UNIT = "tokens/s"
@@ -293,9 +293,29 @@ def run_reference(args, w, rep):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * total / len(times),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": config_of(w, args.gpus),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "cpu": host_cpu(), "kind": "oracle",
+                         "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
+
+
+def host_cpu():
+    """Model name of the host CPU (lscpu, else /proc/cpuinfo), for the oracle's timing record."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith(("model name", "cpu part")):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return None
 
 
 def config_of(w, n_gpus, shard="replicas"):
@@ -533,7 +553,8 @@ def time_prefill(w, q, k, v, steps, warmup, rep, peaks, peak_src, local, min_sec
     total_f = flops.useful_flops(B, Hq, N, d, w.n_sink, w.window, w.gamma)
     useful_tflops = total_f / (ms_per_step / 1e3) / 1e12
     sustained = float(peaks.get("bf16_tflops_sustained", PEAKS_FALLBACK["bf16_tflops_sustained"]))
-    rec = {"ms_per_step": ms_per_step, "timed_repeats": repeats, "loop_ms": loop_ms,
+    rec = {"ms_per_step": ms_per_step, "median_ms_per_step": statistics.median(loop_ms) / steps,
+           "timed_repeats": repeats, "loop_ms": loop_ms,
            "useful_tflops": useful_tflops, "pct_of_bf16_peak": 100 * useful_tflops / peak,
            "pct_of_bf16_sustained": 100 * useful_tflops / sustained, "roofline": roofline, "kernels": kernels,
            "gpu_launches": nk * steps * repeats, "clocks": clock_info}
@@ -573,7 +594,8 @@ def time_workloads(args, dev, rep, peaks, peak_src):
 
     def one(w, q, k, v, dense_reps=0):
         rec, out, _ = time_prefill(w, q, k, v, min(args.steps, 10), 3, rep, peaks, peak_src, rep.local)
-        rec.update({"tokens_per_s": w.B * w.N / (rec["ms_per_step"] / 1e3), "config": config_of(w, 1)})
+        rec.update({"tokens_per_s": w.B * w.N / (rec["ms_per_step"] / 1e3), "config": config_of(w, 1),
+                    "input_checksums": checksums(q, k, v)})
         for key in ("loop_ms",):
             rec.pop(key, None)
         del out
@@ -697,7 +719,8 @@ def run_ours(args, w, rep):
     }
     result.update({key: rec[key] for key in ("useful_tflops", "pct_of_bf16_peak", "pct_of_bf16_sustained",
                                              "roofline", "kernels", "gpu_launches", "clocks", "timed_repeats",
-                                             "loop_ms")})
+                                             "loop_ms", "median_ms_per_step")})
+    result["input_checksums"] = checksums(q, k, v)
     if sharded:
         result["useful_tflops"] = flops.useful_flops(w.B, w.Hq, w.N, w.d, w.n_sink, w.window, w.gamma) / (
             ms_per_step / 1e3) / 1e12
@@ -757,7 +780,7 @@ def run_ours(args, w, rep):
         result["parity"] = parity_spot_check(w, q, k, v, out, Qb, Kb, Vb)
         tps, secs, groups, cores = oracle_sample(w, Qb, Kb, Vb, args.cpu_seconds)
         result["cpu_baseline"] = {
-            "value": tps, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "value": tps, "unit": UNIT, "cores": cores, "cpu": host_cpu(), "kind": "oracle",
             "sample": "%d groups of gamma=%d rows x all %d query heads at evenly spaced positions of the "
                       "%d-token sequence, fp64 C oracle on %d threads, %.1f s" % (
                           groups, w.gamma, w.Hq, w.N, cores, secs)}

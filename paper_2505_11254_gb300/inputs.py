@@ -99,9 +99,19 @@ def generate(w: Workload, device="cpu", N: Optional[int] = None):
     return Q, K, V
 
 
-def checksum(t: torch.Tensor) -> int:
-    """Sum of the bf16 bit patterns as signed 16-bit integers (record keeping)."""
-    return int(t.contiguous().view(torch.int16).to(torch.int64).sum().item())
+def checksum(t: torch.Tensor, chunk: int = 1 << 26) -> int:
+    """Sum of the bf16 bit patterns as signed 16-bit integers (record keeping),
+    taken over slices of `chunk` elements so that no full-size wider copy is
+    made; the same bits give the same value on any device."""
+    flat = t.contiguous().view(-1).view(torch.int16)
+    total = 0
+    for i in range(0, flat.numel(), chunk):
+        total += int(flat[i:i + chunk].to(torch.int64).sum().item())
+    return total
+
+
+def checksums(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor) -> dict:
+    return {"kind": "sum of bf16 bit patterns as int16", "Q": checksum(q), "K": checksum(k), "V": checksum(v)}
 
 
 def to_bits(t: torch.Tensor):
