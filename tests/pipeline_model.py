@@ -1,0 +1,379 @@
+"""An executable model of the attention kernel's synchronisation
+(`csrc/attn_kernel.cuh`), checked by random interleavings on the CPU.
+
+Each warp role is a Python generator that yields the mbarrier wait it is
+about to make, in the kernel's order and with the kernel's phase arithmetic;
+arrivals happen where the kernel arrives.  Two asynchronous engines complete
+work in the background: the tensor pipe (MMAs and tcgen05.commit, in issue
+order) and the copy engine (TMA loads, in any order).  mbarriers follow the
+PTX semantics of `mbarrier.try_wait.parity`: a wait for the phase of parity P
+passes whenever the barrier's current phase has the other parity.  The model
+therefore flags
+
+  * an aliased wait: it passes while the phase it means is not the last one
+    completed (the barrier is a phase behind, or two ahead);
+  * buffer hazards: a copy into a K, V or Q slot, a QK into an S/P buffer, a
+    first PV into O, a row-sum slot, a queue slot or a Q buffer in TMEM reused
+    before its previous reader is done;
+  * deadlock: no role, engine or copy can move.
+
+Two layouts, as in the kernel: the sink + window passes (Q in shared memory,
+three S/P buffers, NQ = 1 at d = 128 or 2 at d = 64, optional RoPE rotation
+of each Q tile by the epilogue warps) and the strided dense pass (Q copied
+into a TMEM double buffer by the epilogue warps, two S/P buffers, work items
+claimed by the producer and published through the eight-slot item queue).
+Thread counts of an arrival (128 softmax or epilogue threads) are modelled as
+one arrival on a barrier of count one."""
+import random
+
+
+class ModelError(Exception):
+    pass
+
+
+class Bar:
+    def __init__(self, name):
+        self.name, self.ph = name, 0
+
+    def arrive(self):
+        self.ph += 1
+
+
+def _check_wait(bar, k):
+    ok = (bar.ph & 1) != (k & 1)
+    if ok and bar.ph != k + 1:
+        raise ModelError("aliased wait on %s: wants phase %d, %d completed" % (bar.name, k, bar.ph))
+    if not ok and bar.ph >= k + 2:
+        raise ModelError("wait on %s for phase %d passed by: %d completed" % (bar.name, k, bar.ph))
+    return ok
+
+
+class Layout:
+    def __init__(self, dense, nq=1, rope=False, nk=3, nv=2):
+        self.dense = dense
+        self.qtmem = dense
+        self.nq = 1 if dense else nq
+        self.nsb = 2 if dense else 3
+        self.nk, self.nv = nk, nv
+        self.rope = rope and not dense
+        self.dyn = dense
+
+
+def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
+    """Run one random interleaving; `tiles` lists each item's key-tile count
+    (the CTA's items in order).  `mutant` names a deliberate protocol error
+    (see MUTANTS) for the checker's own tests."""
+    L, rnd = layout, random.Random(seed)
+    n = len(tiles)
+    bars = {}
+
+    def bar(name):
+        bars[name] = Bar(name)
+        return bars[name]
+
+    kfull = [bar("kfull%d" % s) for s in range(L.nk)]
+    kempty = [bar("kempty%d" % s) for s in range(L.nk)]
+    vfull = [bar("vfull%d" % s) for s in range(L.nv)]
+    vempty = [bar("vempty%d" % s) for s in range(L.nv)]
+    q_full = [bar("q_full%d" % b) for b in range(2)]
+    q_free = [bar("q_free%d" % b) for b in range(2)]
+    qt_ready = [bar("qt_ready%d" % b) for b in range(2)]
+    s_full = [bar("s_full%d" % b) for b in range(L.nsb)]
+    p_full = [bar("p_full%d" % b) for b in range(L.nsb)]
+    pv_done = [bar("pv_done%d" % b) for b in range(L.nsb)]
+    o_full, o_free = bar("o_full"), bar("o_free")
+    l_ready = [bar("l_ready%d" % b) for b in range(2)]
+    l_free = [bar("l_free%d" % b) for b in range(2)]
+    kq = 8
+    iq_full = [bar("iq_full%d" % s) for s in range(kq)]
+    iq_empty_count = [0] * kq  # readers that released each queue slot (one completion = 5 roles)
+    iq_empty = [bar("iq_empty%d" % s) for s in range(kq)]
+    readers = 5  # V producer, QK, PV, softmax, epilogue (each warp group counted once)
+
+    pipe, copies = [], []
+    done = {"qk": set(), "pv": set(), "o_read": set(), "q_rot": set(), "q_copied": set(), "l_read": set(),
+            "iq_read": {}}
+    first_g = []
+    g = 0
+    for T in tiles:
+        first_g.append(g)
+        g += T
+
+    def iq_release(slot):
+        iq_empty_count[slot] += 1
+        if iq_empty_count[slot] == readers:
+            iq_empty_count[slot] = 0
+            iq_empty[slot].arrive()
+
+    class Reader:
+        """The item sequence as a role reads it: static, or from the queue."""
+
+        def __init__(self, name):
+            self.name, self.k = name, 0
+
+        def next(self):
+            if not L.dyn:
+                i = self.k
+                self.k += 1
+                return i if i < n else -1
+            slot = self.k % kq
+            yield (iq_full[slot], self.k // kq)
+            v = done["iq_read"][self.k]
+            iq_release(slot)
+            self.k += 1
+            return v
+
+    def producer():
+        nq = 0
+        c = 0
+        np_ = 0
+        claimed = 0
+
+        def claim():
+            nonlocal np_, claimed
+            v = claimed if claimed < n else -1
+            claimed += 1
+            if L.dyn:
+                slot = np_ % kq
+                if np_ >= kq:
+                    yield (iq_empty[slot], np_ // kq - 1)
+                done["iq_read"][np_] = v
+                iq_full[slot].arrive()
+                np_ += 1
+            return v
+
+        def load_q(item):
+            nonlocal nq
+            qb = nq % L.nq
+            if nq >= L.nq and mutant != "q_no_free_wait":
+                yield (q_free[qb], nq // L.nq - 1)
+            if nq >= L.nq:
+                prev = nq - L.nq
+                if L.qtmem and prev not in done["q_copied"]:
+                    raise ModelError("Q smem buffer reloaded before the epilogue copied Q(%d)" % prev)
+                if not L.qtmem:
+                    last = first_g[prev] + tiles[prev] - 1
+                    if last not in done["qk"]:
+                        raise ModelError("Q buffer reloaded before the last QK of item %d" % prev)
+            copies.append((q_full[qb], ("q", nq)))
+            nq += 1
+
+        item = yield from claim()
+        if item >= 0:
+            yield from load_q(item)
+        while item >= 0:
+            nxt = -1
+            for j in range(tiles[item]):
+                s = c % L.nk
+                if c >= L.nk:
+                    yield (kempty[s], c // L.nk - 1)
+                    if (c - L.nk) not in done["qk"]:
+                        raise ModelError("K slot reloaded before QK(%d) completed" % (c - L.nk))
+                copies.append((kfull[s], ("k", c)))
+                c += 1
+                if j == 0:
+                    nxt = yield from claim()
+                    if (L.nq >= 2 or L.qtmem) and nxt >= 0:
+                        yield from load_q(nxt)
+            if L.nq == 1 and not L.qtmem and nxt >= 0:
+                yield from load_q(nxt)
+            item = nxt
+        if L.dyn and claimed <= n:
+            yield from claim()
+
+    def vprod():
+        rd = Reader("v")
+        c = 0
+        while True:
+            item = yield from rd.next()
+            if item < 0:
+                return
+            for j in range(tiles[item]):
+                s = c % L.nv
+                if c >= L.nv:
+                    yield (vempty[s], c // L.nv - 1)
+                    if (c - L.nv) not in done["pv"]:
+                        raise ModelError("V slot reloaded before PV(%d) completed" % (c - L.nv))
+                copies.append((vfull[s], ("v", c)))
+                c += 1
+
+    def qk():
+        rd = Reader("qk")
+        g = 0
+        i = 0
+        while True:
+            item = yield from rd.next()
+            if item < 0:
+                return
+            qb = (i & 1) if L.qtmem else i % L.nq
+            if L.qtmem or L.rope:
+                yield (qt_ready[qb], (i >> 1) if L.qtmem else i // L.nq)
+            else:
+                yield (q_full[qb], i // L.nq)
+            for j in range(tiles[item]):
+                ks, sbi = g % L.nk, g % L.nsb
+                yield (kfull[ks], g // L.nk)
+                if g >= L.nsb and mutant != "qk_no_pv_wait":
+                    yield (pv_done[sbi], g // L.nsb - 1)
+                pipe.append(("qk", g, item))
+                pipe.append(("commit", s_full[sbi]))
+                g += 1
+            if not L.qtmem:
+                pipe.append(("commit", q_free[qb]))
+            i += 1
+
+    def pv():
+        rd = Reader("pv")
+        g = 0
+        i = 0
+        while True:
+            item = yield from rd.next()
+            if item < 0:
+                return
+            T = tiles[item]
+            for j in range(T):
+                vs, sbi = g % L.nv, g % L.nsb
+                yield (p_full[sbi], g // L.nsb)
+                yield (vfull[vs], g // L.nv)
+                if j == 0 and i >= 1 and mutant != "pv_no_o_free":
+                    yield (o_free, i - 1)
+                pipe.append(("pv", g, item, j == 0))
+                pipe.append(("commit", pv_done[sbi]))
+                pipe.append(("commit", vempty[vs]))
+                if j == T - 1:
+                    pipe.append(("commit", o_full))
+                g += 1
+            i += 1
+
+    def softmax():
+        rd = Reader("softmax")
+        g = 0
+        i = 0
+        while True:
+            item = yield from rd.next()
+            if item < 0:
+                return
+            for j in range(tiles[item]):
+                sbi = g % L.nsb
+                yield (s_full[sbi], g // L.nsb)
+                if g not in done["qk"]:
+                    raise ModelError("softmax read S(%d) before its QK completed" % g)
+                kempty[g % L.nk].arrive()
+                if j >= 1 and rnd.random() < rescale_p:  # lazy O rescale: PV(g-1) must have landed
+                    yield (pv_done[(g - 1) % L.nsb], (g - 1) // L.nsb)
+                    if (g - 1) not in done["pv"]:
+                        raise ModelError("O rescaled before PV(%d) completed" % (g - 1))
+                p_full[sbi].arrive()
+                yield None
+                g += 1
+            if i >= 2 and mutant != "softmax_no_l_free":
+                yield (l_free[i & 1], (i >> 1) - 1)
+            if i >= 2 and (i - 2) not in done["l_read"]:
+                raise ModelError("row sums of item %d overwritten before the epilogue read them" % (i - 2))
+            l_ready[i & 1].arrive()
+            i += 1
+
+    def epilogue():
+        rd = Reader("epilogue")
+        nq = 0
+
+        def rotate(buf, qi):
+            nonlocal nq
+            if L.qtmem:
+                yield (q_full[0], nq)
+                nq += 1
+                # TMEM buffer buf last held the Q of item qi - 2, read by its QKs
+                if qi >= 2:
+                    last = first_g[qi - 2] + tiles[qi - 2] - 1
+                    if last not in done["qk"]:
+                        raise ModelError("TMEM Q buffer rewritten before the QKs of item %d completed" % (qi - 2))
+                done["q_copied"].add(qi)
+                qt_ready[buf].arrive()
+                q_free[0].arrive()
+            elif L.rope:
+                yield (q_full[buf], nq // L.nq)
+                nq += 1
+                done["q_rot"].add(qi)
+                qt_ready[buf].arrive()
+
+        item = yield from rd.next()
+        if item >= 0:
+            yield from rotate(0, 0)
+        i = 0
+        while item >= 0:
+            nxt = yield from rd.next()
+            if nxt >= 0:
+                yield from rotate(((i + 1) & 1) if L.qtmem else (i + 1) % L.nq, i + 1)
+            yield (l_ready[i & 1], i >> 1)
+            done["l_read"].add(i)
+            l_free[i & 1].arrive()
+            yield (o_full, i + 1 if mutant == "o_full_phase_ahead" else i)
+            done["o_read"].add(i)
+            o_free.arrive()
+            item = nxt
+            i += 1
+
+    roles = {"producer": producer(), "vprod": vprod(), "qk": qk(), "pv": pv(), "softmax": softmax(),
+             "epilogue": epilogue()}
+    waits = {}
+    finished = set()
+
+    def advance(name):
+        try:
+            waits[name] = next(roles[name])
+        except StopIteration:
+            finished.add(name)
+            waits[name] = None
+
+    for name in roles:
+        advance(name)
+    # each actor gets a random speed for this run, so that some runs starve
+    # one role (a slow epilogue, a slow copy engine) and others the next
+    speed = {name: rnd.choice([0.05, 0.3, 1.0, 1.0, 3.0]) for name in list(roles) + ["pipe", "copy"]}
+    for _ in range(max_steps):
+        cands = []
+        for name in roles:
+            if name in finished:
+                continue
+            w = waits[name]
+            if w is None or _check_wait(*w):
+                cands.append(("role", name))
+        if pipe:
+            cands.append(("pipe", None))
+        if copies:
+            cands.append(("copy", None))
+        if not cands:
+            if len(finished) == len(roles):
+                return
+            raise ModelError("deadlock: " + "; ".join(
+                "%s waits %s for phase %d (%d completed)" % (nm, waits[nm][0].name, waits[nm][1], waits[nm][0].ph)
+                for nm in roles if nm not in finished and waits[nm] is not None))
+        kind, name = rnd.choices(cands, weights=[speed[c[1] if c[0] == "role" else c[0]] for c in cands])[0]
+        if kind == "role":
+            advance(name)
+        elif kind == "pipe":
+            op = pipe.pop(0)
+            if op[0] == "qk":
+                gg, item = op[1], op[2]
+                if gg >= L.nsb and (gg - L.nsb) not in done["pv"]:
+                    raise ModelError("QK(%d) overwrote S/P buffer before PV(%d) read it" % (gg, gg - L.nsb))
+                if L.rope and item not in done["q_rot"]:
+                    raise ModelError("QK of item %d read Q before its rotation" % item)
+                done["qk"].add(gg)
+            elif op[0] == "pv":
+                gg, item, first = op[1], op[2], op[3]
+                if first and item >= 1 and (item - 1) not in done["o_read"]:
+                    raise ModelError("first PV of item %d overwrote O before item %d's was read" % (item, item - 1))
+                done["pv"].add(gg)
+            else:
+                op[1].arrive()
+        else:
+            b, _ = copies.pop(rnd.randrange(len(copies)))
+            b.arrive()
+    raise ModelError("no end after %d steps" % max_steps)
+
+
+# Each drops or misaims one wait of the protocol above.  The last waits for
+# the next phase of o_full: with the barrier one phase behind, the parity
+# test passes at once (the aliasing that a parity wait must never meet).
+MUTANTS = ["qk_no_pv_wait", "pv_no_o_free", "softmax_no_l_free", "q_no_free_wait", "o_full_phase_ahead"]

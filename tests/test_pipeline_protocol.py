@@ -1,0 +1,54 @@
+"""The attention kernel's barrier protocol, run as an executable model over
+random interleavings (`pipeline_model.py`): no parity wait may pass on the
+wrong phase, no buffer may be refilled before its reader is done, and every
+interleaving must finish.  Covered: the sink + window layout at d = 128 and
+d = 64 (one or two Q buffers), with and without the RoPE rotation of each Q
+tile, and the strided dense layout (Q in TMEM, items through the queue).
+Item lengths include one- and two-tile items and the long items of wide
+windows, so the ring and buffer indices wrap at every offset.  Deliberately
+broken protocols (a dropped wait each) must be caught, which shows that the
+model sees what it is meant to."""
+import random
+
+import pytest
+
+from pipeline_model import MUTANTS, Layout, ModelError, run
+
+LAYOUTS = {
+    "sink_window_d128": Layout(dense=False, nq=1),
+    "sink_window_d64": Layout(dense=False, nq=2, nk=4, nv=4),
+    "sink_window_d128_rope": Layout(dense=False, nq=1, rope=True),
+    "sink_window_d64_rope": Layout(dense=False, nq=2, nk=4, nv=4, rope=True),
+    "strided_dense_d128": Layout(dense=True),
+    "strided_dense_d64": Layout(dense=True, nk=4, nv=4),
+}
+
+
+def _items(rnd):
+    return [rnd.choice([1, 1, 2, 3, 4, 5, 6, 7, 18]) for _ in range(rnd.randint(0, 9))]
+
+
+@pytest.mark.parametrize("name", sorted(LAYOUTS))
+def test_protocol_holds_over_random_interleavings(name):
+    rnd = random.Random(hash(name) & 0xffff)
+    for r in range(300):
+        tiles = _items(rnd)
+        try:
+            run(LAYOUTS[name], tiles, seed=r)
+        except ModelError as e:
+            pytest.fail("%s, items %s, seed %d: %s" % (name, tiles, r, e))
+
+
+@pytest.mark.parametrize("mutant", MUTANTS)
+def test_a_dropped_wait_is_caught(mutant):
+    layouts = ([LAYOUTS["strided_dense_d128"], LAYOUTS["sink_window_d128"]] if mutant == "q_no_free_wait"
+               else [LAYOUTS["sink_window_d128"], LAYOUTS["strided_dense_d128"]])
+    rnd = random.Random(7)
+    for r in range(400):
+        tiles = _items(rnd) + [18, 3]
+        for lay in layouts:
+            try:
+                run(lay, tiles, seed=r, mutant=mutant)
+            except ModelError:
+                return
+    pytest.fail("mutant %s was not caught" % mutant)
