@@ -12,13 +12,13 @@
 //              aliasing S); lazy O rescaling; per item the row sum l and max m.
 //   warps 4-7  epilogue: rotates the next item's Q in smem ahead of time when
 //              RoPE is on, then reads O out of TMEM, releases it, normalises,
-//              applies the Delta correction and writes the output.
+//              applies the Delta correction (or, in the dense pass, writes or
+//              merges the split-K partials) and writes the output.
 //   warp 8     TMA producer: Q of the next item, K tiles through their ring.
 //   warp 9     QK issuer: S = Q K^T once its K tile has landed and the PV
-//              that last read the S buffer has completed.  Sink + window
-//              passes: Q from smem (one buffer at d = 128, reloaded after the
-//              item's last QK; two at d = 64).  Dense pass: Q from TMEM
-//              (two buffers, filled by the epilogue warps).
+//              that last read the S buffer has completed; Q and K from smem
+//              (one Q buffer at d = 128, reloaded after the item's last QK;
+//              two at d = 64).
 //   warp 10    PV issuer: O += P V (P from TMEM, V from smem) once the softmax
 //              has written P(g).  Two issuing threads keep the tensor pipe fed:
 //              neither waits on the other's inputs.
@@ -27,10 +27,9 @@
 // Registers: launched at 168 per thread (384 x 168 = 64512); the third
 // warpgroup gives back to 72 and the softmax and epilogue warpgroups grow to
 // 216, so 2 x 128 x 216 + 128 x 72 = 64512 exactly.
-// TMEM (512 columns), two layouts (see Cfg): sink + window passes hold an
-// S/P triple buffer and O, so QK may run three tiles ahead of the softmax and
-// the chain softmax(g) -> PV(g) -> QK(g+3) spans three tiles; the dense pass
-// holds Q (two buffers), an S/P double buffer and O.
+// TMEM (512 columns, see Cfg): an S/P triple buffer and O, so QK may run
+// three tiles ahead of the softmax and the chain softmax(g) -> PV(g) ->
+// QK(g+3) spans three tiles.
 // Every wait is bounded: past its limit a wait sets the CTA's abort flag and
 // the device status word, the roles stop working (keeping every named barrier
 // and warp-collective instruction uniform), drain their in-flight copies and
@@ -59,29 +58,25 @@ static_assert(2 * 128 * kRegsCompute + 128 * kRegsControl <= kThreads * 168, "re
 constexpr float RESCALE_THRESHOLD = 64.0f;
 constexpr uint32_t kFull = 0xffffffffu;
 
-// Two TMEM layouts (512 columns):
-//   Q in TMEM (the dense pass): Q double buffer [0,64) [64,128) (bf16 pairs),
-//     S/P double buffer [128,256) [256,384), O [384, 384 + D); QK reads Q from
-//     TMEM, so a tile's shared-memory traffic is its K and V only;
-//   Q in smem (the sink + window passes): S/P triple buffer [0,128) [128,256)
-//     [256,384), O [384, 384 + D); QK reads Q and K from smem and may run
-//     three tiles ahead of the softmax.
+// TMEM layout (512 columns), all passes: S/P triple buffer [0,128) [128,256)
+// [256,384), O [384, 384 + D).  QK reads Q and K from smem and may run three
+// tiles ahead of the softmax.  (A dense-pass layout with Q in TMEM, two S/P
+// buffers and no Q reads from smem measured 6-7 % slower: the third S buffer
+// is worth more than the shared-memory reads it saves.)
 template <int D, int MODE = MODE_SPARSE>
 struct Cfg {
-  static constexpr bool QTMEM = (MODE == MODE_STRIDED_DENSE);
-  static constexpr int NQ = (D == 128 || QTMEM) ? 1 : 2;  // Q buffers in smem
+  static constexpr int NQ = (D == 128) ? 1 : 2;           // Q buffers in smem
   static constexpr int NK = (D == 128) ? 3 : 4;           // K ring slots (D = 128: five fit beside Q)
   static constexpr int NV = (D == 128) ? 2 : 4;           // V ring slots
   static constexpr int NS = NK + NV;
-  static constexpr int NSB = QTMEM ? 2 : 3;               // S/P buffers in TMEM
+  static constexpr int NSB = 3;                           // S/P buffers in TMEM
   static constexpr int CHUNKS = D / 64;          // 64-element (128-byte) swizzle columns
   static constexpr uint32_t Q_BYTES = BM * D * 2;
   static constexpr uint32_t KV_BYTES = BN * D * 2;
   static constexpr uint32_t SBUF_BYTES = kSampleBufBytes;  // sampled sparse rows of the fused epilogue
   static constexpr uint32_t SMEM = NQ * Q_BYTES + NS * KV_BYTES + SBUF_BYTES + 1024;
   static constexpr uint32_t TMEM_COLS = 512;
-  static constexpr uint32_t COL_Q = 0;                  // + 64 * buffer (Q in TMEM)
-  static constexpr uint32_t COL_S = QTMEM ? 128 : 0;    // + BN * buffer
+  static constexpr uint32_t COL_S = 0;                  // + BN * buffer
   static constexpr uint32_t COL_O = 384;
   static constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, 0, 0);
   static constexpr uint32_t IDESC_PV = idesc_bf16(BM, D, 0, 1);
@@ -263,7 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bars.q_full[b], 1);
-      mbar_init(&bars.q_free[b], C::QTMEM ? 128 : 1);  // the epilogue's copy, or the last QK
+      mbar_init(&bars.q_free[b], 1);  // the item's last QK
       mbar_init(&bars.qt_ready[b], 128);
       mbar_init(&bars.l_ready[b], 128);
       mbar_init(&bars.l_free[b], 128);
@@ -362,13 +357,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = load_k(krow, kz);
           if (ok && j == 0) {
             nxt = claim();
-            // with two Q buffers, or Q copied to TMEM, the next item's Q goes out at once
-            if ((C::NQ >= 2 || C::QTMEM) && nxt >= 0) ok = load_q(nxt);
+            // with two Q buffers the next item's Q goes out at once
+            if (C::NQ >= 2 && nxt >= 0) ok = load_q(nxt);
           }
         }
         // with one Q buffer it waits for this item's last QK, so it goes out
         // after this item's K/V loads (which that QK needs)
-        if (C::NQ == 1 && !C::QTMEM && ok && nxt >= 0) ok = load_q(nxt);
+        if (C::NQ == 1 && ok && nxt >= 0) ok = load_q(nxt);
         item = nxt;
       }
       if (DYN && !done) claim();  // the readers always see the end of the sequence
@@ -392,15 +387,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       int i = 0;
       for (long long item = items.next(p, iq, &abort_sh); ok && item >= 0; item = items.next(p, iq, &abort_sh), ++i) {
         const Work w = decode_work<MODE, ROWS>(p, item);
-        // Q of item i: in TMEM buffer i & 1 (copied by the epilogue), or in smem
-        // buffer i % NQ (rotated in place first when RoPE is on)
-        const int qb = C::QTMEM ? (i & 1) : i % C::NQ;
-        uint64_t* qbar = (C::QTMEM || rope) ? &bars.qt_ready[qb] : &bars.q_full[qb];
-        if (!wait_bounded(qbar, (uint32_t)(C::QTMEM ? (i >> 1) : i / C::NQ) & 1, &abort_sh, p.err)) {
+        // Q of item i: in smem buffer i % NQ (rotated in place first when RoPE is on)
+        const int qb = i % C::NQ;
+        uint64_t* qbar = rope ? &bars.qt_ready[qb] : &bars.q_full[qb];
+        if (!wait_bounded(qbar, (uint32_t)(i / C::NQ) & 1, &abort_sh, p.err)) {
           ok = false;
           break;
         }
-        const uint32_t qt = tmem + C::COL_Q + (uint32_t)qb * 64;
         const uint64_t qd = qdesc0 + ((qb * C::Q_BYTES) >> 4);
         for (int j = 0; j < w.T; ++j, ++g) {
           const int ks = (int)(g % C::NK);
@@ -419,14 +412,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint32_t off = (((kk >> 2) * (BN * 128)) + (kk & 3) * 32) >> 4;
-            if (C::QTMEM)
-              mma_ts(sb, qt + kk * 8, kd + off, C::IDESC_QK, kk > 0 ? 1u : 0u);
-            else
-              mma_ss(sb, qd + off, kd + off, C::IDESC_QK, kk > 0 ? 1u : 0u);
+            mma_ss(sb, qd + off, kd + off, C::IDESC_QK, kk > 0 ? 1u : 0u);
           }
           mma_commit(&bars.s_full[sbi]);
         }
-        if (!C::QTMEM && ok) mma_commit(&bars.q_free[qb]);  // the item's last QK has read its Q
+        if (ok) mma_commit(&bars.q_free[qb]);  // the item's last QK has read its Q
       }
       if (!ok)  // after an early exit, read the item queue to its end marker
         while (items.next(p, iq, &abort_sh) >= 0) {}
@@ -634,67 +624,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t la = lane_base(warp);
     bool ok = true;
     int nq = 0;
-    // Q of an item: swizzled smem rows -> TMEM lanes (bf16 pairs), the A
-    // operand of S = Q K^T.
     // RoPE (Sec. 2), rotate-half, when Q comes unrotated: each row of the
     // item's Q tile turns in place in its smem buffer before its first QK.
     // Channel c turns with channel c + D/2 by the angle of the row's position;
     // word k of r holds channels 2k and 2k + 1, its partner word is k + D/4.
     // fp32, one rounding to bf16.  Without RoPE the QK reads the TMA'd tile.
-    // Q in TMEM: the item's Q tile, swizzled smem rows -> TMEM lanes (bf16
-    // pairs), rotated on the way when RoPE is on; frees the smem buffer.
-    auto copy_q = [&](int buf, long long qitem) {
-      ok = ok && __all_sync(kFull, wait_sleepy(&bars.q_full[0], nq & 1, &abort_sh, p.err));
-      ++nq;
-      if (ok) {
-        uint32_t r[D / 2];
-#pragma unroll
-        for (int ch = 0; ch < C::CHUNKS; ++ch)
-#pragma unroll
-          for (int pc = 0; pc < 8; ++pc) {
-            const uint4 v =
-                *reinterpret_cast<const uint4*>(sQ + ch * (BM * 128) + e * 128 + ((pc ^ (e & 7)) * 16));
-            r[ch * 32 + pc * 4 + 0] = v.x;
-            r[ch * 32 + pc * 4 + 1] = v.y;
-            r[ch * 32 + pc * 4 + 2] = v.z;
-            r[ch * 32 + pc * 4 + 3] = v.w;
-          }
-        if (p.rope != nullptr) {
-          const Work wq = decode_work<MODE, ROWS>(p, qitem);
-          long long qrow, qsample;
-          int qhead;
-          if (lane_row<MODE>(p, wq, e, qrow, qsample, qhead)) {
-            const float4* cs = reinterpret_cast<const float4*>(p.rope + qrow * D);
-#pragma unroll
-            for (int k = 0; k < D / 4; ++k) {
-              const float4 t = __ldg(cs + k);  // (cos, sin) of channels 2k, 2k + 1
-              const float a0 = __uint_as_float(r[k] << 16), a1 = __uint_as_float(r[k] & 0xffff0000u);
-              const float b0 = __uint_as_float(r[k + D / 4] << 16);
-              const float b1 = __uint_as_float(r[k + D / 4] & 0xffff0000u);
-              r[k] = pack_bf16x2(a0 * t.x - b0 * t.y, a1 * t.z - b1 * t.w);
-              r[k + D / 4] = pack_bf16x2(b0 * t.x + a0 * t.y, b1 * t.z + a1 * t.w);
-            }
-          }
-        }
-#pragma unroll
-        for (int q = 0; q < D / 64; ++q) {
-          uint32_t rr[32];
-#pragma unroll
-          for (int c = 0; c < 32; ++c) rr[c] = r[q * 32 + c];
-          tmem_st32(tmem + la + C::COL_Q + buf * 64 + q * 32, rr);
-        }
-        tmem_st_wait();
-      }
-      fence_proxy_async_smem();  // the next TMA write of sQ follows these reads
-      tc_fence_before();
-      mbar_arrive(&bars.qt_ready[buf]);
-      mbar_arrive(&bars.q_free[0]);
-    };
     auto rotate_q = [&](int buf, long long qitem) {
-      if (C::QTMEM) {
-        copy_q(buf, qitem);
-        return;
-      }
       if (p.rope == nullptr) return;
       ok = ok && __all_sync(kFull, wait_sleepy(&bars.q_full[buf], (nq / C::NQ) & 1, &abort_sh, p.err));
       ++nq;
@@ -741,7 +676,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; item >= 0; ++i) {
       const Work w = decode_work<MODE, ROWS>(p, item);
       const long long nxt = items.next(p, iq, &abort_sh);
-      if (nxt >= 0) rotate_q(C::QTMEM ? ((i + 1) & 1) : (i + 1) % C::NQ, nxt);
+      if (nxt >= 0) rotate_q((i + 1) % C::NQ, nxt);
       long long row, sample;
       int head;
       const bool row_ok = lane_row<MODE>(p, w, e, row, sample, head);

@@ -7,8 +7,8 @@
 //   * rope_apply_kernel: rotates bf16 rows in place (K before the prefill, a
 //     decode query at its position): HBM-bound, 16-byte coalesced accesses,
 //     fp32 arithmetic, one rounding to bf16.
-// Q is not rotated here: the attention kernels rotate each Q tile while
-// copying it into tensor memory (EPI warps, copy_q), saving a read and a
+// Q is not rotated here: the attention kernels rotate each Q tile in shared
+// memory before its first QK (epilogue warps, rotate_q), saving a read and a
 // write of Q.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>

@@ -13,15 +13,15 @@ therefore flags
   * an aliased wait: it passes while the phase it means is not the last one
     completed (the barrier is a phase behind, or two ahead);
   * buffer hazards: a copy into a K, V or Q slot, a QK into an S/P buffer, a
-    first PV into O, a row-sum slot, a queue slot or a Q buffer in TMEM reused
-    before its previous reader is done;
+    first PV into O, a row-sum slot or a queue slot reused before its previous
+    reader is done, a QK reading a Q tile before its rotation;
   * deadlock: no role, engine or copy can move.
 
-Two layouts, as in the kernel: the sink + window passes (Q in shared memory,
-three S/P buffers, NQ = 1 at d = 128 or 2 at d = 64, optional RoPE rotation
-of each Q tile by the epilogue warps) and the strided dense pass (Q copied
-into a TMEM double buffer by the epilogue warps, two S/P buffers, work items
-claimed by the producer and published through the eight-slot item queue).
+Both passes share the layout (Q in shared memory, three S/P buffers, NQ = 1
+at d = 128 or 2 at d = 64, optional RoPE rotation of each Q tile by the
+epilogue warps); the sink + window passes walk a static item sequence, the
+strided dense pass claims its items in the producer and publishes them
+through the eight-slot item queue.
 Thread counts of an arrival (128 softmax or epilogue threads) are modelled as
 one arrival on a barrier of count one."""
 import random
@@ -50,13 +50,8 @@ def _check_wait(bar, k):
 
 class Layout:
     def __init__(self, dense, nq=1, rope=False, nk=3, nv=2):
-        self.dense = dense
-        self.qtmem = dense
-        self.nq = 1 if dense else nq
-        self.nsb = 2 if dense else 3
-        self.nk, self.nv = nk, nv
-        self.rope = rope and not dense
-        self.dyn = dense
+        self.dyn = dense  # items through the queue
+        self.nq, self.nsb, self.nk, self.nv, self.rope = nq, 3, nk, nv, rope
 
 
 def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
@@ -91,8 +86,7 @@ def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
     readers = 5  # V producer, QK, PV, softmax, epilogue (each warp group counted once)
 
     pipe, copies = [], []
-    done = {"qk": set(), "pv": set(), "o_read": set(), "q_rot": set(), "q_copied": set(), "l_read": set(),
-            "iq_read": {}}
+    done = {"qk": set(), "pv": set(), "o_read": set(), "q_rot": set(), "l_read": set(), "iq_read": {}}
     first_g = []
     g = 0
     for T in tiles:
@@ -149,12 +143,9 @@ def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
                 yield (q_free[qb], nq // L.nq - 1)
             if nq >= L.nq:
                 prev = nq - L.nq
-                if L.qtmem and prev not in done["q_copied"]:
-                    raise ModelError("Q smem buffer reloaded before the epilogue copied Q(%d)" % prev)
-                if not L.qtmem:
-                    last = first_g[prev] + tiles[prev] - 1
-                    if last not in done["qk"]:
-                        raise ModelError("Q buffer reloaded before the last QK of item %d" % prev)
+                last = first_g[prev] + tiles[prev] - 1
+                if last not in done["qk"]:
+                    raise ModelError("Q buffer reloaded before the last QK of item %d" % prev)
             copies.append((q_full[qb], ("q", nq)))
             nq += 1
 
@@ -173,9 +164,9 @@ def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
                 c += 1
                 if j == 0:
                     nxt = yield from claim()
-                    if (L.nq >= 2 or L.qtmem) and nxt >= 0:
+                    if L.nq >= 2 and nxt >= 0:
                         yield from load_q(nxt)
-            if L.nq == 1 and not L.qtmem and nxt >= 0:
+            if L.nq == 1 and nxt >= 0:
                 yield from load_q(nxt)
             item = nxt
         if L.dyn and claimed <= n:
@@ -205,11 +196,8 @@ def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
             item = yield from rd.next()
             if item < 0:
                 return
-            qb = (i & 1) if L.qtmem else i % L.nq
-            if L.qtmem or L.rope:
-                yield (qt_ready[qb], (i >> 1) if L.qtmem else i // L.nq)
-            else:
-                yield (q_full[qb], i // L.nq)
+            qb = i % L.nq
+            yield (qt_ready[qb] if L.rope else q_full[qb], i // L.nq)
             for j in range(tiles[item]):
                 ks, sbi = g % L.nk, g % L.nsb
                 yield (kfull[ks], g // L.nk)
@@ -218,8 +206,7 @@ def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
                 pipe.append(("qk", g, item))
                 pipe.append(("commit", s_full[sbi]))
                 g += 1
-            if not L.qtmem:
-                pipe.append(("commit", q_free[qb]))
+            pipe.append(("commit", q_free[qb]))
             i += 1
 
     def pv():
@@ -279,18 +266,7 @@ def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
 
         def rotate(buf, qi):
             nonlocal nq
-            if L.qtmem:
-                yield (q_full[0], nq)
-                nq += 1
-                # TMEM buffer buf last held the Q of item qi - 2, read by its QKs
-                if qi >= 2:
-                    last = first_g[qi - 2] + tiles[qi - 2] - 1
-                    if last not in done["qk"]:
-                        raise ModelError("TMEM Q buffer rewritten before the QKs of item %d completed" % (qi - 2))
-                done["q_copied"].add(qi)
-                qt_ready[buf].arrive()
-                q_free[0].arrive()
-            elif L.rope:
+            if L.rope:
                 yield (q_full[buf], nq // L.nq)
                 nq += 1
                 done["q_rot"].add(qi)
@@ -303,7 +279,7 @@ def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
         while item >= 0:
             nxt = yield from rd.next()
             if nxt >= 0:
-                yield from rotate(((i + 1) & 1) if L.qtmem else (i + 1) % L.nq, i + 1)
+                yield from rotate((i + 1) % L.nq, i + 1)
             yield (l_ready[i & 1], i >> 1)
             done["l_read"].add(i)
             l_free[i & 1].arrive()

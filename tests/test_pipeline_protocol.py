@@ -3,7 +3,7 @@ random interleavings (`pipeline_model.py`): no parity wait may pass on the
 wrong phase, no buffer may be refilled before its reader is done, and every
 interleaving must finish.  Covered: the sink + window layout at d = 128 and
 d = 64 (one or two Q buffers), with and without the RoPE rotation of each Q
-tile, and the strided dense layout (Q in TMEM, items through the queue).
+tile, and the strided dense pass (the same layout, items through the queue).
 Item lengths include one- and two-tile items and the long items of wide
 windows, so the ring and buffer indices wrap at every offset.  Deliberately
 broken protocols (a dropped wait each) must be caught, which shows that the
@@ -20,7 +20,8 @@ LAYOUTS = {
     "sink_window_d128_rope": Layout(dense=False, nq=1, rope=True),
     "sink_window_d64_rope": Layout(dense=False, nq=2, nk=4, nv=4, rope=True),
     "strided_dense_d128": Layout(dense=True),
-    "strided_dense_d64": Layout(dense=True, nk=4, nv=4),
+    "strided_dense_d64": Layout(dense=True, nq=2, nk=4, nv=4),
+    "strided_dense_d128_rope": Layout(dense=True, rope=True),
 }
 
 
