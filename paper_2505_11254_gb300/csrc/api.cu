@@ -294,7 +294,7 @@ int check_decode(int B, int Hq, int Hkv, int64_t L, int64_t max_keys, int d) {
 
 DecodePlan make_decode_plan(int B, int Hq, int Hkv, int64_t max_keys, int d, int sms) {
   DecodePlan dp;
-  const long long chunk = decode_keys_per_split();
+  const long long chunk = decode_keys_per_split(d, Hq / Hkv);
   const long long chunks = cdiv(max_keys, chunk);
   const long long pairs = (long long)B * Hkv;
   // at most one wave: a second, partial wave would run alone at the end

@@ -7,9 +7,12 @@
 // (with one query row per head there is no tile to fill).  Design:
 //   * split-K: a CTA per (batch, KV head, key range) handles the G query
 //     heads of the KV group together, so each K/V byte is read once;
-//   * a producer warp streams 32-key K and V chunks (contiguous rows) with
-//     cp.async.bulk into a 4-stage shared-memory ring completed on mbarriers;
-//     the key range is split so that one wave of CTAs fills every SM;
+//   * a producer warp streams K and V chunks (contiguous rows) with
+//     cp.async.bulk into a shared-memory ring completed on mbarriers: eight
+//     stages of 16 keys (two per consumer warp, so a warp's next chunk loads
+//     while it works on the current one) or, when a warp iteration takes 32
+//     keys, four of 32; the key range is split so that one wave of CTAs fills
+//     every SM;
 //   * four consumer warps take whole chunks in turn.  Inside a warp, groups
 //     of LPK lanes work on different keys (layout in DecLayout): a lane holds
 //     a slice of the channels of q and o for every head (GP = G rounded up to
@@ -35,20 +38,8 @@ namespace {
 
 constexpr int kDecWarps = 4;                        // consumer warps
 constexpr int kDecThreads = (kDecWarps + 1) * 32;   // + the producer warp
-constexpr int kDecChunk = 32;                       // keys per ring stage
-constexpr int kDecStages = 4;
 constexpr int kDecQORegs = 64;  // registers per lane for its slices of q and o
 constexpr int kDecMinCtas = 2;  // CTAs per SM the register allocation must allow
-// Chunk i goes to stage i % kDecStages and to consumer warp i % kDecWarps.
-// With kDecStages a multiple of kDecWarps every phase of a stage is consumed
-// by the same warp in order, so a parity wait can never be satisfied by a
-// phase two behind the one it wants.
-static_assert(kDecStages % kDecWarps == 0, "each stage must belong to one consumer warp");
-
-template <int D>
-constexpr int dec_smem_bytes() {
-  return kDecStages * 2 * kDecChunk * D * 2 + 1024;
-}
 
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
@@ -95,7 +86,22 @@ struct DecLayout {
   static constexpr int PS = CPL < 8 ? CPL : 8;   // channels per piece
   static constexpr int T = CPL / PS;             // pieces per lane
   static_assert(KG >= 1 && N % GP == 0 && N % LPK == 0, "layout");
-  static_assert(kDecChunk % KEYS == 0, "a chunk holds whole iterations");
+};
+
+// The ring of a kernel instance: chunks of max(16, KEYS) keys, eight stages
+// of 16 keys or four of 32 (64 KB at d = 128 either way, so two CTAs fit an
+// SM).  Chunk i goes to stage i % STAGES and to consumer warp i % kDecWarps.
+// With STAGES a multiple of kDecWarps every phase of a stage is consumed by
+// the same warp in order, so a parity wait can never be satisfied by a phase
+// two behind the one it wants.
+template <int D, int GP>
+struct DecRing {
+  static constexpr int KEYS = DecLayout<D, GP>::KEYS;
+  static constexpr int CHUNK = KEYS > 16 ? KEYS : 16;
+  static constexpr int STAGES = CHUNK == 16 ? 8 : 4;
+  static constexpr int SMEM = STAGES * 2 * CHUNK * D * 2 + 1024;
+  static_assert(CHUNK % KEYS == 0, "a chunk holds whole iterations");
+  static_assert(STAGES % kDecWarps == 0, "each stage must belong to one consumer warp");
 };
 
 // Channels of one row slice (T pieces of PS channels) as floats.
@@ -131,12 +137,14 @@ __device__ __forceinline__ void load_slice(const __nv_bfloat16* row, int sub, fl
 template <int D, int GP>
 __global__ void __launch_bounds__(kDecThreads, kDecMinCtas) decode_kernel(DecodeParams p) {
   using L = DecLayout<D, GP>;
+  using Ring = DecRing<D, GP>;
   constexpr int CPL = L::CPL, R = L::R, LPK = L::LPK, KG = L::KG, N = L::N;
+  constexpr int CHUNK = Ring::CHUNK, STAGES = Ring::STAGES;  // keys per stage, stages
   constexpr unsigned kFull = 0xffffffffu;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __nv_bfloat16* ring = reinterpret_cast<__nv_bfloat16*>(smem);  // [stage][K|V][kDecChunk][D]
-  __shared__ uint64_t full[kDecStages], empty[kDecStages];
+  __nv_bfloat16* ring = reinterpret_cast<__nv_bfloat16*>(smem);  // [stage][K|V][CHUNK][D]
+  __shared__ uint64_t full[STAGES], empty[STAGES];
   __shared__ volatile int abort_sh;
   constexpr int kStates = kDecWarps * L::NG;  // (warp, group) partial softmax states
   __shared__ float sm_m[kStates][GP], sm_l[kStates][GP];
@@ -151,12 +159,12 @@ __global__ void __launch_bounds__(kDecThreads, kDecMinCtas) decode_kernel(Decode
   n = n < 0 ? 0 : (n > p.L ? p.L : n);
   const long long k_begin = (long long)s * p.split_keys;
   const long long k_end = (k_begin + p.split_keys < n) ? k_begin + p.split_keys : n;
-  const int nc = k_end > k_begin ? (int)((k_end - k_begin + kDecChunk - 1) / kDecChunk) : 0;
+  const int nc = k_end > k_begin ? (int)((k_end - k_begin + CHUNK - 1) / CHUNK) : 0;
 
   if (threadIdx.x == 0) {
     // let the merge grid be scheduled now; it waits for this grid's completion
     asm volatile("griddepcontrol.launch_dependents;");
-    for (int i = 0; i < kDecStages; ++i) {
+    for (int i = 0; i < STAGES; ++i) {
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 1);
     }
@@ -172,20 +180,20 @@ __global__ void __launch_bounds__(kDecThreads, kDecMinCtas) decode_kernel(Decode
     if (lane == 0) {
       int issued = 0;
       for (int i = 0; i < nc; ++i) {
-        const int st = i % kDecStages;
-        if (i >= kDecStages && !wait_bounded(&empty[st], ((i / kDecStages) - 1) & 1, &abort_sh, p.err)) break;
-        const long long k0 = k_begin + (long long)i * kDecChunk;
-        const long long nk = (k_end - k0 < kDecChunk) ? k_end - k0 : kDecChunk;
+        const int st = i % STAGES;
+        if (i >= STAGES && !wait_bounded(&empty[st], ((i / STAGES) - 1) & 1, &abort_sh, p.err)) break;
+        const long long k0 = k_begin + (long long)i * CHUNK;
+        const long long nk = (k_end - k0 < CHUNK) ? k_end - k0 : CHUNK;
         const uint32_t bytes = (uint32_t)(nk * D * 2);
         mbar_arrive_expect_tx(&full[st], 2 * bytes);
-        bulk_g2s(ring + (size_t)(st * 2) * kDecChunk * D, Kg + k0 * D, bytes, &full[st]);
-        bulk_g2s(ring + (size_t)(st * 2 + 1) * kDecChunk * D, Vg + k0 * D, bytes, &full[st]);
+        bulk_g2s(ring + (size_t)(st * 2) * CHUNK * D, Kg + k0 * D, bytes, &full[st]);
+        bulk_g2s(ring + (size_t)(st * 2 + 1) * CHUNK * D, Vg + k0 * D, bytes, &full[st]);
         ++issued;
       }
       // The ring must be quiet before the CTA exits: wait for the latest
       // phase of every stage still in use.
-      for (int i = (issued > kDecStages ? issued - kDecStages : 0); i < issued; ++i)
-        wait_drain(&full[i % kDecStages], (i / kDecStages) & 1, p.err);
+      for (int i = (issued > STAGES ? issued - STAGES : 0); i < issued; ++i)
+        wait_drain(&full[i % STAGES], (i / STAGES) & 1, p.err);
     }
     return;
   }
@@ -220,13 +228,13 @@ __global__ void __launch_bounds__(kDecThreads, kDecMinCtas) decode_kernel(Decode
   const int kk_own = (sub * R) / GP;  // key (within the group's KG) of this lane's scores
 
   for (int i = warp; i < nc; i += kDecWarps) {
-    const int st = i % kDecStages;
-    if (!__all_sync(kFull, wait_bounded(&full[st], (i / kDecStages) & 1, &abort_sh, p.err))) break;
-    const __nv_bfloat16* Ks = ring + (size_t)(st * 2) * kDecChunk * D;
-    const __nv_bfloat16* Vs = ring + (size_t)(st * 2 + 1) * kDecChunk * D;
-    const long long k0 = k_begin + (long long)i * kDecChunk;
-    const int nk = (int)((k_end - k0 < kDecChunk) ? k_end - k0 : kDecChunk);
-    const bool partial = nk < kDecChunk;  // warp-uniform
+    const int st = i % STAGES;
+    if (!__all_sync(kFull, wait_bounded(&full[st], (i / STAGES) & 1, &abort_sh, p.err))) break;
+    const __nv_bfloat16* Ks = ring + (size_t)(st * 2) * CHUNK * D;
+    const __nv_bfloat16* Vs = ring + (size_t)(st * 2 + 1) * CHUNK * D;
+    const long long k0 = k_begin + (long long)i * CHUNK;
+    const int nk = (int)((k_end - k0 < CHUNK) ? k_end - k0 : CHUNK);
+    const bool partial = nk < CHUNK;  // warp-uniform
 #pragma unroll 1
     for (int kb = 0; kb < nk; kb += L::KEYS) {
       const int key0 = kb + grp * KG;  // this group's first key in the chunk
@@ -441,11 +449,11 @@ cudaError_t launch_decode_t(const DecodeParams& p, long long units, cudaStream_t
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64 || !attr_set[dev]) {
-    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, dec_smem_bytes<D>());
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, DecRing<D, GP>::SMEM);
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) attr_set[dev] = true;
   }
-  k<<<(unsigned)units, kDecThreads, dec_smem_bytes<D>(), s>>>(p);
+  k<<<(unsigned)units, kDecThreads, DecRing<D, GP>::SMEM, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -461,7 +469,16 @@ cudaError_t launch_decode_d(const DecodeParams& p, long long units, cudaStream_t
 
 }  // namespace
 
-int decode_keys_per_split() { return kDecChunk; }
+template <int D>
+int keys_per_chunk_d(int G) {
+  if (G <= 1) return DecRing<D, 1>::CHUNK;
+  if (G <= 2) return DecRing<D, 2>::CHUNK;
+  if (G <= 4) return DecRing<D, 4>::CHUNK;
+  if (G <= 8) return DecRing<D, 8>::CHUNK;
+  return DecRing<D, 16>::CHUNK;
+}
+
+int decode_keys_per_split(int d, int G) { return d == 64 ? keys_per_chunk_d<64>(G) : keys_per_chunk_d<128>(G); }
 
 // Queried once per kernel instance (the answer is the same on every GB300;
 // concurrent first calls compute the same value).
@@ -471,8 +488,8 @@ int ctas_per_sm_t() {
   if (cached > 0) return cached;
   int n = 0;
   auto k = decode_kernel<D, GP>;
-  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, dec_smem_bytes<D>()) != cudaSuccess ||
-      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, kDecThreads, dec_smem_bytes<D>()) != cudaSuccess)
+  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, DecRing<D, GP>::SMEM) != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k, kDecThreads, DecRing<D, GP>::SMEM) != cudaSuccess)
     return 1;
   cached = n > 0 ? n : 1;
   return cached;

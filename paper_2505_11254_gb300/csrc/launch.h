@@ -33,12 +33,12 @@ struct DecodeParams {
   long long max_keys, L;
   int B, Hq, Hkv, G, D;
   int n_split;             // key ranges per (batch, KV head)
-  long long split_keys;    // keys per range, a multiple of decode_keys_per_split()
+  long long split_keys;    // keys per range, a multiple of decode_keys_per_split(d, G)
   float scale_log2;        // log2(e) / sqrt(D)
   float* part;             // [B * Hkv * n_split][G][D + 2]: unnormalised o, max, sum
   int* err;                // device status word
 };
-int decode_keys_per_split();
+int decode_keys_per_split(int d, int G);  // keys per ring chunk of the kernel instance
 int decode_ctas_per_sm(int d, int G);  // resident decode CTAs per SM (occupancy)
 cudaError_t launch_decode(const DecodeParams& p, void* out, cudaStream_t s);
 
