@@ -353,3 +353,66 @@ def run(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
 # the next phase of o_full: with the barrier one phase behind, the parity
 # test passes at once (the aliasing that a parity wait must never meet).
 MUTANTS = ["qk_no_pv_wait", "pv_no_o_free", "softmax_no_l_free", "q_no_free_wait", "o_full_phase_ahead"]
+
+
+def run_decode_ring(n_chunks, stages, warps, seed):
+    """The decode kernel's ring (`csrc/decode.cu`): one producer thread loads
+    chunk i into stage i % stages after the consumer of chunk i - stages
+    released it; consumer warp w takes chunks w, w + warps, ... and waits for
+    chunk i on stage i % stages with the parity of phase i / stages.  The
+    kernel requires stages % warps == 0 so that every phase of a stage is
+    consumed by one warp in order; the model flags the aliased waits
+    otherwise."""
+    rnd = random.Random(seed)
+    full = [Bar("full%d" % s) for s in range(stages)]
+    empty = [Bar("empty%d" % s) for s in range(stages)]
+    in_stage, consumed, pending = {}, set(), []
+
+    def producer():
+        for i in range(n_chunks):
+            st = i % stages
+            if i >= stages:
+                yield (empty[st], i // stages - 1)
+                if (i - stages) not in consumed:
+                    raise ModelError("stage %d reloaded before chunk %d was consumed" % (st, i - stages))
+            pending.append((st, i))
+
+    def consumer(w):
+        for i in range(w, n_chunks, warps):
+            st = i % stages
+            yield (full[st], i // stages)
+            if in_stage.get(st) != i:
+                raise ModelError("warp %d read stage %d for chunk %d, found %s" % (w, st, i, in_stage.get(st)))
+            consumed.add(i)
+            yield None
+            empty[st].arrive()
+
+    roles = {"producer": producer()}
+    roles.update({"warp%d" % w: consumer(w) for w in range(warps)})
+    waits, finished = {}, set()
+
+    def advance(name):
+        try:
+            waits[name] = next(roles[name])
+        except StopIteration:
+            finished.add(name)
+            waits[name] = None
+
+    for name in roles:
+        advance(name)
+    speed = {name: rnd.choice([0.1, 1.0, 3.0]) for name in list(roles) + ["copy"]}
+    while True:
+        cands = [nm for nm in roles if nm not in finished and (waits[nm] is None or _check_wait(*waits[nm]))]
+        if pending:
+            cands.append("copy")
+        if not cands:
+            if len(finished) == len(roles):
+                return
+            raise ModelError("deadlock in the decode ring")
+        name = rnd.choices(cands, weights=[speed[c] for c in cands])[0]
+        if name == "copy":
+            st, i = pending.pop(rnd.randrange(len(pending)))
+            in_stage[st] = i
+            full[st].arrive()
+        else:
+            advance(name)

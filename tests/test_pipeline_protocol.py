@@ -7,12 +7,14 @@ tile, and the strided dense pass (the same layout, items through the queue).
 Item lengths include one- and two-tile items and the long items of wide
 windows, so the ring and buffer indices wrap at every offset.  Deliberately
 broken protocols (a dropped wait each) must be caught, which shows that the
-model sees what it is meant to."""
+model sees what it is meant to.  The decode kernel's K/V ring is checked the
+same way: the deployed eight- and four-stage rings over four consumer warps
+pass, a six-stage ring (stages shared between warps) must be flagged."""
 import random
 
 import pytest
 
-from pipeline_model import MUTANTS, Layout, ModelError, run
+from pipeline_model import MUTANTS, Layout, ModelError, run, run_decode_ring
 
 LAYOUTS = {
     "sink_window_d128": Layout(dense=False, nq=1),
@@ -53,3 +55,26 @@ def test_a_dropped_wait_is_caught(mutant):
             except ModelError:
                 return
     pytest.fail("mutant %s was not caught" % mutant)
+
+
+@pytest.mark.parametrize("stages, warps", [(8, 4), (4, 4)])
+def test_decode_ring_holds(stages, warps):
+    rnd = random.Random(stages * 31 + warps)
+    for r in range(500):
+        n = rnd.randint(0, 40)
+        try:
+            run_decode_ring(n, stages, warps, seed=r)
+        except ModelError as e:
+            pytest.fail("%d stages, %d warps, %d chunks, seed %d: %s" % (stages, warps, n, r, e))
+
+
+def test_decode_ring_with_shared_stages_is_caught():
+    """Six stages over four warps: a stage's phases alternate between warps,
+    so a parity wait can pass on a phase two behind."""
+    rnd = random.Random(3)
+    for r in range(500):
+        try:
+            run_decode_ring(rnd.randint(8, 40), 6, 4, seed=r)
+        except ModelError:
+            return
+    pytest.fail("the shared-stage ring was not caught")
