@@ -299,8 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       auto load_q = [&](long long item) {
         const Work wq = decode_work<MODE, ROWS>(p, item);
-        // buffer qb held the Q of item nq - NQ: its last QK (or, Q in TMEM, the
-        // epilogue's copy) must have read it
+        // buffer qb held the Q of item nq - NQ: its last QK must have read it
         const int qb = nq % C::NQ;
         if (nq >= C::NQ && !wait_bounded(&bars.q_free[qb], ((nq / C::NQ) - 1) & 1, &abort_sh, p.err)) return false;
         mbar_arrive_expect_tx(&bars.q_full[qb], C::Q_BYTES);
