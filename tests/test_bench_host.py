@@ -1,7 +1,8 @@
 """bench.py host logic without a GPU: the kernel-source hash that decides
 whether the recorded ncu DRAM traffic belongs to the kernels being timed
 ignores comments and whitespace-only lines but follows every code change, and
-a record is reported only for the code and workload it was taken on."""
+a record is reported only for the code and workload it was taken on, and the
+input checksums do not depend on how the sum is sliced."""
 import importlib.util
 import json
 import os
@@ -45,3 +46,19 @@ def test_recorded_traffic_lookup():
         want = e["dram_bytes_per_launch"] if e["src_sha"] == sha else None
         assert b.recorded_traffic(name, e["workload"]) == want
         assert b.recorded_traffic(name, "another_workload") is None
+
+
+def test_input_checksums_are_chunk_independent():
+    """The bench records a checksum of each generated bf16 tensor, summed in
+    slices so that no full-size wider copy is made: any slice size gives the
+    sum of the bit patterns as 16-bit integers."""
+    import torch
+    from paper_2505_11254_gb300.inputs import TINY_N2048, checksum, checksums, generate
+    g = torch.Generator().manual_seed(0)
+    x = torch.randn(10007, generator=g).to(torch.bfloat16)
+    ref = int(x.view(torch.int16).to(torch.int64).sum())
+    assert all(checksum(x, chunk=c) == ref for c in (1, 7, 4096, 1 << 26))
+    q, k, v = generate(TINY_N2048)
+    rec = checksums(q, k, v)
+    assert rec["Q"] == checksum(q) and rec["K"] == checksum(k) and rec["V"] == checksum(v)
+    assert generate(TINY_N2048)[0].equal(q), "seeded generation is repeatable"
