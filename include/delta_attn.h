@@ -31,6 +31,13 @@
  * address is looked up once per device, on the first launching call made with
  * that device current.  Results are deterministic: fixed merge order, no
  * floating-point atomics.
+ *
+ * Kernel choice: the sink + window pass of a whole sequence at d = 128 with
+ * an even Hq / Hkv and window >= 2048 runs as a two-CTA kernel (thread-block
+ * clusters of two, one per pair of query heads of a KV group); other shapes
+ * run the one-CTA kernel.  Both give the same bits.  The environment variable
+ * DELTA_ATTN_PAIR, read at each call, overrides the choice: "0" always takes
+ * the one-CTA kernel, "1" the two-CTA kernel wherever the shape allows it.
  */
 #ifndef DELTA_ATTN_H
 #define DELTA_ATTN_H

@@ -14,8 +14,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libdeltaattn.so")
-SOURCES = ["api.cu", "aux.cu", "attn_sparse.cu", "attn_dense.cu", "attn_strided_sparse.cu", "attn_smooth.cu",
-           "smooth.cu", "decode.cu", "rope.cu", "host_pipeline.cu", "noalloc.cu", "attn_rows.cu"]
+SOURCES = ["api.cu", "aux.cu", "attn_sparse.cu", "attn_sparse_pair.cu", "attn_dense.cu", "attn_strided_sparse.cu",
+           "attn_smooth.cu", "smooth.cu", "decode.cu", "rope.cu", "host_pipeline.cu", "noalloc.cu", "attn_rows.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-I" + INCLUDE, "-I" + CSRC]

@@ -7,6 +7,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstdlib>
 #include <mutex>
 
 #include "delta_attn.h"
@@ -198,7 +199,26 @@ int status_ptr(int** ptr) {
 
 struct Maps {
   CUtensorMap q, qs, k, v;
+  CUtensorMap kh;  // K in boxes of BN / 2 rows: the two-CTA sink + window kernel (pair_sparse)
 };
+
+// The sink + window pass of a whole sequence runs as the two-CTA kernel when
+// the query heads of each KV group pair up (G even) at d = 128 and the window
+// spans at least 16 key tiles.  Measured on GB300 against the one-CTA kernel:
+// the same time per prefill at windows 2048 and 8192 (at a higher sustained
+// clock under the power cap: it moves half the K/V bytes through each SM's
+// shared memory and from L2), 2-3 % slower at window 512, whose 6-tile items
+// pay the pair's cross-CTA item hand-off more often.  Results are
+// bit-identical.  The environment variable DELTA_ATTN_PAIR overrides the
+// choice: 0 always takes the one-CTA kernel, 1 the two-CTA one where it
+// applies.
+bool pair_sparse(int d, const Params& p) {
+  if (d != 128 || p.G % 2 != 0 || p.q_row0 != 0) return false;
+  const char* env = getenv("DELTA_ATTN_PAIR");
+  if (env != nullptr && env[0] == '0') return false;
+  if (env != nullptr && env[0] == '1') return true;
+  return p.window >= 16 * BN;
+}
 
 // Sampled rows row0 + k * gamma of every (b, head): Hp heads x R samples a box.
 // Q holds rows q_row0 .. N - 1 of every (b, head); sample k is row row0 + k gamma.
@@ -219,6 +239,9 @@ bool make_maps(Maps* m, const void* Q, const void* K, const void* V, const Param
   if (need_samples && !make_sample_map(&m->qs, Q, p, d)) return false;
   if (!make_map(&m->k, K, d, n_kv, row_bytes, (long long)p.B * p.Hkv, n_kv * row_bytes, BN, 1)) return false;
   if (!make_map(&m->v, V, d, n_kv, row_bytes, (long long)p.B * p.Hkv, n_kv * row_bytes, BN, 1)) return false;
+  if (need_rows && pair_sparse(d, p) &&
+      !make_map(&m->kh, K, d, n_kv, row_bytes, (long long)p.B * p.Hkv, n_kv * row_bytes, BN / 2, 1))
+    return false;
   return true;
 }
 
@@ -229,14 +252,19 @@ cudaError_t launch(int d, const CUtensorMap& q, const CUtensorMap& k, const CUte
   return launch_attn<128, MODE, EPI>(q, k, v, p, grid, s);
 }
 
-// The sink + window pass of a row-range call: the ROWS instance when the range
-// starts after row 0.
+// The sink + window pass: the two-CTA kernel where pair_sparse() allows it,
+// the ROWS instance for a row-range call whose range starts after row 0, the
+// one-CTA whole-sequence kernel otherwise.
 template <int EPI>
-cudaError_t launch_sparse(int d, const CUtensorMap& q, const CUtensorMap& k, const CUtensorMap& v, const Params& p,
-                          long long grid, cudaStream_t s) {
-  if (p.q_row0 == 0) return launch<MODE_SPARSE, EPI>(d, q, k, v, p, grid, s);
-  if (d == 64) return launch_attn<64, MODE_SPARSE, EPI, true>(q, k, v, p, grid, s);
-  return launch_attn<128, MODE_SPARSE, EPI, true>(q, k, v, p, grid, s);
+cudaError_t launch_sparse(int d, const Maps& m, const Params& p, long long grid, cudaStream_t s) {
+  if (pair_sparse(d, p)) return launch_attn<128, MODE_SPARSE, EPI, false, true>(m.q, m.kh, m.v, p, grid, s);
+  if (p.q_row0 == 0) return launch<MODE_SPARSE, EPI>(d, m.q, m.k, m.v, p, grid, s);
+  // Row ranges are Eq. 6 prefills only (delta_attn_prefill_rows).
+  if constexpr (EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA) {
+    if (d == 64) return launch_attn<64, MODE_SPARSE, EPI, true>(m.q, m.k, m.v, p, grid, s);
+    return launch_attn<128, MODE_SPARSE, EPI, true>(m.q, m.k, m.v, p, grid, s);
+  }
+  return cudaErrorInvalidValue;
 }
 
 class ScopedWorkspace {
@@ -514,7 +542,7 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
     p.out_bf16 = O_abs;
     p.smooth_basis = basis - s_off * kSmoothJ * d;  // kSmoothJ vectors per sample
     p.smooth_coef = coef;
-    e = launch<MODE_SPARSE, EPI_FUSED_SMOOTH>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+    e = launch_sparse<EPI_FUSED_SMOOTH>(d, m, p, pl.grid_sparse, s);
     if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
     return run_tail();
   }
@@ -528,7 +556,7 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
     // Eq. 5: sparse rows everywhere, then the sampled rows overwritten by
     // their dense rows; no correction reaches the other rows.
     p.out_bf16 = O_abs;
-    e = launch<MODE_SPARSE, EPI_BF16>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+    e = launch_sparse<EPI_BF16>(d, m, p, pl.grid_sparse, s);
     if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
     e = launch<MODE_STRIDED_DENSE, EPI_DENSE_BF16>(d, m.qs, m.k, m.v, p, pl.grid_dense, s);
     if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
@@ -542,7 +570,7 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
   p.out_bf16 = O_abs;
   if (pl.fused_intile) {
     p.d_in = abs_samples(dbuf);
-    e = launch_sparse<EPI_FUSED_INTILE>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+    e = launch_sparse<EPI_FUSED_INTILE>(d, m, p, pl.grid_sparse, s);
   } else {
     float* delta = reinterpret_cast<float*>(base + pl.off_delta);
     p.d_in = dbuf;  // the strided sparse pass indexes its own samples
@@ -552,7 +580,7 @@ static int prefill_impl(const void* Q, const void* K, const void* V, void* O, in
     p.delta_out = nullptr;
     p.d_in = abs_samples(dbuf);
     p.delta_in = abs_samples(delta);
-    e = launch_sparse<EPI_FUSED_DELTA>(d, m.q, m.k, m.v, p, pl.grid_sparse, s);
+    e = launch_sparse<EPI_FUSED_DELTA>(d, m, p, pl.grid_sparse, s);
   }
   if (e != cudaSuccess || !mark()) return DA_ERR_CUDA;
   return run_tail();
@@ -609,7 +637,7 @@ int sparse_window_attn(const void* Q, const void* K, const void* V, void* O_spar
   if (!make_maps(&m, Q, K, V, p, d, true, false, N)) return DA_ERR_INVALID_ARG;
   p.out_bf16 = O_sparse;
   p.s_sampled = S_sampled;
-  cudaError_t e = launch<MODE_SPARSE, EPI_BF16>(d, m.q, m.k, m.v, p, pl.grid_sparse, static_cast<cudaStream_t>(stream));
+  cudaError_t e = launch_sparse<EPI_BF16>(d, m, p, pl.grid_sparse, static_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? DA_OK : DA_ERR_CUDA;
 }
 

@@ -63,29 +63,46 @@ constexpr uint32_t kFull = 0xffffffffu;
 // tiles ahead of the softmax.  (A dense-pass layout with Q in TMEM, two S/P
 // buffers and no Q reads from smem measured 6-7 % slower: the third S buffer
 // is worth more than the shared-memory reads it saves.)
-template <int D, int MODE = MODE_SPARSE>
+//
+// PAIR (sink + window pass, d = 128, the query heads of a KV group taken two
+// at a time): a cluster of two CTAs runs the two heads' items of the same
+// row tile, which visit the same key tiles.  The leader issues every MMA for
+// both with cta_group::2 (M = 256): each CTA keeps its own Q, S/P and O, and
+// holds only half of each K tile (keys 0-63 in the leader, 64-127 in the peer)
+// and half of each V tile (columns 0-63 / 64-127).  Per tile an SM then moves
+// 96 KB through shared memory (Q 32, K half 16 and V half 16 read by the
+// tensor core, 32 written by TMA) instead of 160 KB.
+template <int D, int MODE = MODE_SPARSE, bool PAIR = false>
 struct Cfg {
-  static constexpr int NQ = (D == 128) ? 1 : 2;           // Q buffers in smem
-  static constexpr int NK = (D == 128) ? 3 : 4;           // K ring slots (D = 128: five fit beside Q)
-  static constexpr int NV = (D == 128) ? 2 : 4;           // V ring slots
+  static_assert(!PAIR || (D == 128 && MODE == MODE_SPARSE), "the two-CTA form is the d = 128 sink + window pass");
+  static constexpr int NQ = PAIR ? 2 : (D == 128) ? 1 : 2;  // Q buffers in smem
+  static constexpr int NK = PAIR ? 5 : (D == 128) ? 3 : 4;  // K ring slots (D = 128: five fit beside Q)
+  static constexpr int NV = PAIR ? 4 : (D == 128) ? 2 : 4;  // V ring slots
   static constexpr int NS = NK + NV;
   static constexpr int NSB = 3;                           // S/P buffers in TMEM
   static constexpr int CHUNKS = D / 64;          // 64-element (128-byte) swizzle columns
   static constexpr uint32_t Q_BYTES = BM * D * 2;
-  static constexpr uint32_t KV_BYTES = BN * D * 2;
+  static constexpr uint32_t K_BYTES = (PAIR ? BN / 2 : BN) * D * 2;  // a K slot: this CTA's keys of a tile
+  static constexpr uint32_t V_BYTES = BN * (PAIR ? D / 2 : D) * 2;   // a V slot: this CTA's columns of a tile
+  static constexpr uint32_t K_CHUNK = (PAIR ? BN / 2 : BN) * 128;    // bytes of one swizzle column of a K slot
+  static constexpr int V_CHUNKS = PAIR ? 1 : CHUNKS;
   static constexpr uint32_t SBUF_BYTES = kSampleBufBytes;  // sampled sparse rows of the fused epilogue
-  static constexpr uint32_t SMEM = NQ * Q_BYTES + NS * KV_BYTES + SBUF_BYTES + 1024;
+  static constexpr uint32_t SMEM = NQ * Q_BYTES + NK * K_BYTES + NV * V_BYTES + SBUF_BYTES + 1024;
   static constexpr uint32_t TMEM_COLS = 512;
   static constexpr uint32_t COL_S = 0;                  // + BN * buffer
   static constexpr uint32_t COL_O = 384;
-  static constexpr uint32_t IDESC_QK = idesc_bf16(BM, BN, 0, 0);
-  static constexpr uint32_t IDESC_PV = idesc_bf16(BM, D, 0, 1);
+  static constexpr uint32_t IDESC_QK = idesc_bf16(PAIR ? 2 * BM : BM, BN, 0, 0);
+  static constexpr uint32_t IDESC_PV = idesc_bf16(PAIR ? 2 * BM : BM, D, 0, 1);
+  // Arrivals that complete p_full, o_free and qt_ready: every thread of the
+  // warpgroup, or in a pair one per warp of both CTAs.
+  static constexpr uint32_t ARRIVALS = PAIR ? 8 : 128;
   static_assert(COL_O + D <= TMEM_COLS, "TMEM layout");
+  static_assert(NK <= 8 && NV <= 8, "ring barriers");
   static_assert(SMEM <= 232448, "shared memory above the 227 KB per-block limit");
 };
 
 struct Bars {
-  uint64_t kfull[4], kempty[4], vfull[4], vempty[4];
+  uint64_t kfull[8], kempty[8], vfull[8], vempty[8];
   uint64_t q_full[2], q_free[2];
   uint64_t qt_ready[2];
   uint64_t s_full[3], p_full[3];
@@ -223,18 +240,22 @@ struct ItemReader {
 // ROWS: the kernel of a row-range call (Params::q_row0 > 0): items start at
 // row q_row0, Q and O hold rows from q_row0.  Whole-sequence launches use
 // ROWS = false.
-template <int D, int MODE, int EPI, bool ROWS = false>
+// PAIR: launched in clusters of two (see Cfg).  The items of CTA x are those
+// of the one-CTA kernel (x, x + gridDim.x, ...); with G even and the grid
+// even, items 2c and 2c + 1 are the two heads of one row tile, so the two
+// CTAs of a cluster always work on the same row tile and key tiles.
+template <int D, int MODE, int EPI, bool ROWS = false, bool PAIR = false>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                 const __grid_constant__ CUtensorMap tmV, const Params p) {
-  using C = Cfg<D, MODE>;
-  constexpr int NS = C::NS;
+  using C = Cfg<D, MODE, PAIR>;
+  static_assert(!PAIR || !ROWS, "row-range calls use the one-CTA kernel");
   extern __shared__ uint8_t dsm_raw[];
   uint8_t* dsm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = dsm;  // [NQ][Q_BYTES]: item i uses buffer i % NQ
   uint8_t* ring = sQ + C::NQ * C::Q_BYTES;  // K slots [0, NK), then V slots
-  uint8_t* vring = ring + C::NK * C::KV_BYTES;
-  float* sbuf = reinterpret_cast<float*>(ring + NS * C::KV_BYTES);
+  uint8_t* vring = ring + C::NK * C::K_BYTES;
+  float* sbuf = reinterpret_cast<float*>(vring + C::NV * C::V_BYTES);
 
   __shared__ Bars bars;
   __shared__ uint32_t tmem_base_sh;
@@ -246,6 +267,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
+  // Pair: this CTA's rank; the leader (rank 0) issues the MMAs and owns the
+  // barriers both CTAs signal, addressed through the cluster window.
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  const bool leader = rank == 0;
+  auto at_leader = [&](uint64_t* bar) { return mapa_shared(smem_u32(bar), 0); };
 
   if (tid == 0) {
     for (int s = 0; s < C::NK; ++s) {
@@ -259,17 +285,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bars.q_full[b], 1);
       mbar_init(&bars.q_free[b], 1);  // the item's last QK
-      mbar_init(&bars.qt_ready[b], 128);
+      mbar_init(&bars.qt_ready[b], C::ARRIVALS);
       mbar_init(&bars.l_ready[b], 128);
       mbar_init(&bars.l_free[b], 128);
     }
     for (int b = 0; b < C::NSB; ++b) {
       mbar_init(&bars.s_full[b], 1);
-      mbar_init(&bars.p_full[b], 128);
+      mbar_init(&bars.p_full[b], C::ARRIVALS);
       mbar_init(&bars.pv_done[b], 1);
     }
     mbar_init(&bars.o_full, 1);
-    mbar_init(&bars.o_free, 128);
+    mbar_init(&bars.o_free, C::ARRIVALS);
     mbar_init(&bars.drain, 1);
     mbar_init(&bars.drain2, 1);
     for (int k = 0; k < kQueue; ++k) {
@@ -280,11 +306,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
   }
   if (warp == 0) {
-    tmem_alloc(&tmem_base_sh, C::TMEM_COLS);
-    tmem_relinquish();
+    if (PAIR) {
+      tmem_alloc_pair(&tmem_base_sh, C::TMEM_COLS);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(&tmem_base_sh, C::TMEM_COLS);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   __syncthreads();
+  if (PAIR) cluster_sync();  // both CTAs' barriers exist before either signals the other's
   tc_fence_after();
   const uint32_t tmem = tmem_base_sh;
 
@@ -301,11 +333,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         const Work wq = decode_work<MODE, ROWS>(p, item);
         // buffer qb held the Q of item nq - NQ: its last QK must have read it
         const int qb = nq % C::NQ;
-        if (nq >= C::NQ && !wait_bounded(&bars.q_free[qb], ((nq / C::NQ) - 1) & 1, &abort_sh, p.err)) return false;
-        mbar_arrive_expect_tx(&bars.q_full[qb], C::Q_BYTES);
-        for (int ch = 0; ch < C::CHUNKS; ++ch)
-          tma_load_3d(sQ + qb * C::Q_BYTES + ch * (BM * 128), &tmQ, &bars.q_full[qb], ch * 64,
-                      (int)(ROWS && MODE == MODE_SPARSE ? wq.r0 - p.q_row0 : wq.r0), wq.b * p.Hq + wq.h0);
+        if (nq >= C::NQ && !wait_bounded(&bars.q_free[qb], ((nq / C::NQ) - 1) & 1, &abort_sh, p.err))
+          return false;
+        if (PAIR) {
+          // Without RoPE the QK issuer waits for both CTAs' Q on the leader's
+          // barrier; with RoPE each CTA's epilogue first rotates its own Q.
+          const bool at_lead = p.rope == nullptr;
+          if (leader || !at_lead) mbar_arrive_expect_tx(&bars.q_full[qb], at_lead ? 2 * C::Q_BYTES : C::Q_BYTES);
+          const uint32_t bar = at_lead ? at_leader(&bars.q_full[qb]) : mapa_shared(smem_u32(&bars.q_full[qb]), rank);
+          for (int ch = 0; ch < C::CHUNKS; ++ch)
+            tma_load_3d_pair(sQ + qb * C::Q_BYTES + ch * (BM * 128), &tmQ, bar, ch * 64, (int)wq.r0,
+                             wq.b * p.Hq + wq.h0);
+        } else {
+          mbar_arrive_expect_tx(&bars.q_full[qb], C::Q_BYTES);
+          for (int ch = 0; ch < C::CHUNKS; ++ch)
+            tma_load_3d(sQ + qb * C::Q_BYTES + ch * (BM * 128), &tmQ, &bars.q_full[qb], ch * 64,
+                        (int)(ROWS && MODE == MODE_SPARSE ? wq.r0 - p.q_row0 : wq.r0), wq.b * p.Hq + wq.h0);
+        }
         ++nq;
         return true;
       };
@@ -314,9 +358,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto load_k = [&](int row, int z) {
         const int s = c % C::NK;
         if (c >= C::NK && !wait_bounded(&bars.kempty[s], ((c / C::NK) - 1) & 1, &abort_sh, p.err)) return false;
-        mbar_arrive_expect_tx(&bars.kfull[s], C::KV_BYTES);
-        for (int ch = 0; ch < C::CHUNKS; ++ch)
-          tma_load_3d(ring + s * C::KV_BYTES + ch * (BN * 128), &tmK, &bars.kfull[s], ch * 64, row, z);
+        if (PAIR) {
+          // this CTA's half of the tile's keys, counted on the leader's barrier
+          if (leader) mbar_arrive_expect_tx(&bars.kfull[s], 2 * C::K_BYTES);
+          const uint32_t bar = at_leader(&bars.kfull[s]);
+          for (int ch = 0; ch < C::CHUNKS; ++ch)
+            tma_load_3d_pair(ring + s * C::K_BYTES + ch * C::K_CHUNK, &tmK, bar, ch * 64, row + (int)rank * (BN / 2),
+                             z);
+        } else {
+          mbar_arrive_expect_tx(&bars.kfull[s], C::K_BYTES);
+          for (int ch = 0; ch < C::CHUNKS; ++ch)
+            tma_load_3d(ring + s * C::K_BYTES + ch * C::K_CHUNK, &tmK, &bars.kfull[s], ch * 64, row, z);
+        }
         ++c;
         return true;
       };
@@ -367,14 +420,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (DYN && !done) claim();  // the readers always see the end of the sequence
       // Drain: only the last NK K loads and the last Q loads can be in flight.
-      for (int u = (c > C::NK ? c - C::NK : 0); u < c; ++u) wait_drain(&bars.kfull[u % C::NK], (u / C::NK) & 1, p.err);
-      for (int k = (nq > C::NQ ? nq - C::NQ : 0); k < nq; ++k)
-        wait_drain(&bars.q_full[k % C::NQ], (k / C::NQ) & 1, p.err);
+      // In a pair the leader's barriers count both CTAs' copies, so the leader
+      // drains for both (the peer drains its own Q only when it has a barrier
+      // of its own, with RoPE).
+      if (!PAIR || leader)
+        for (int u = (c > C::NK ? c - C::NK : 0); u < c; ++u)
+          wait_drain(&bars.kfull[u % C::NK], (u / C::NK) & 1, p.err);
+      if (!PAIR || leader || p.rope != nullptr)
+        for (int k = (nq > C::NQ ? nq - C::NQ : 0); k < nq; ++k)
+          wait_drain(&bars.q_full[k % C::NQ], (k / C::NQ) & 1, p.err);
     }
   } else if (warp == 9) {
     // ================================================================ QK issuer
     regs_decrease<kRegsControl>();
-    if ((tid & 31) == 0) {
+    if ((tid & 31) == 0 && leader) {
       // Shared-memory descriptors of Q buffer 0 and ring slot 0; a buffer,
       // slot or K-step adds its byte offset / 16 to the start-address field.
       const uint64_t qdesc0 = sdesc_sw128(smem_u32(sQ), 16, 1024);
@@ -407,25 +466,40 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
           const uint32_t sb = tmem + C::COL_S + (uint32_t)sbi * BN;
-          const uint64_t kd = kdesc0 + ((ks * C::KV_BYTES) >> 4);
+          const uint64_t kd = kdesc0 + ((ks * C::K_BYTES) >> 4);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t off = (((kk >> 2) * (BN * 128)) + (kk & 3) * 32) >> 4;
-            mma_ss(sb, qd + off, kd + off, C::IDESC_QK, kk > 0 ? 1u : 0u);
+            const uint32_t qoff = (((kk >> 2) * (BM * 128)) + (kk & 3) * 32) >> 4;
+            const uint32_t koff = (((kk >> 2) * C::K_CHUNK) + (kk & 3) * 32) >> 4;
+            if (PAIR)
+              mma_ss_pair(sb, qd + qoff, kd + koff, C::IDESC_QK, kk > 0 ? 1u : 0u);
+            else
+              mma_ss(sb, qd + qoff, kd + koff, C::IDESC_QK, kk > 0 ? 1u : 0u);
           }
-          mma_commit(&bars.s_full[sbi]);
+          if (PAIR)
+            mma_commit_pair_both(&bars.s_full[sbi]);
+          else
+            mma_commit(&bars.s_full[sbi]);
         }
-        if (ok) mma_commit(&bars.q_free[qb]);  // the item's last QK has read its Q
+        if (ok) {  // the item's last QK has read its Q
+          if (PAIR)
+            mma_commit_pair_both(&bars.q_free[qb]);
+          else
+            mma_commit(&bars.q_free[qb]);
+        }
       }
       if (!ok)  // after an early exit, read the item queue to its end marker
         while (items.next(p, iq, &abort_sh) >= 0) {}
-      mma_commit(&bars.drain);
+      if (PAIR)
+        mma_commit_pair_local(&bars.drain);
+      else
+        mma_commit(&bars.drain);
       wait_drain(&bars.drain, 0, p.err);
     }
   } else if (warp == 10) {
     // ================================================================ PV issuer
     regs_decrease<kRegsControl>();
-    if ((tid & 31) == 0) {
+    if ((tid & 31) == 0 && leader) {
       const uint64_t vdesc0 = sdesc_sw128(smem_u32(vring), BN * 128, 1024);
       long long g = 0;
       bool ok = true;
@@ -437,25 +511,44 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int vs = (int)(g % C::NV);
           const uint32_t vph = (uint32_t)(g / C::NV) & 1;
           const int sbi = (int)(g % C::NSB);
-          if (!wait_bounded(&bars.p_full[sbi], (uint32_t)(g / C::NSB) & 1, &abort_sh, p.err)) { ok = false; break; }
+          if (!wait_bounded(&bars.p_full[sbi], (uint32_t)(g / C::NSB) & 1, &abort_sh, p.err)) {
+            ok = false;
+            break;
+          }
           if (!wait_bounded(&bars.vfull[vs], vph, &abort_sh, p.err)) { ok = false; break; }
           // The epilogue must have read the previous item's O.
-          if (j == 0 && i >= 1 && !wait_bounded(&bars.o_free, (i - 1) & 1, &abort_sh, p.err)) { ok = false; break; }
+          if (j == 0 && i >= 1 && !wait_bounded(&bars.o_free, (i - 1) & 1, &abort_sh, p.err)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
           const uint32_t sb = tmem + C::COL_S + (uint32_t)sbi * BN;
-          const uint64_t vd = vdesc0 + ((vs * C::KV_BYTES) >> 4);
-          mma_ts(tmem + C::COL_O, sb, vd, C::IDESC_PV, j == 0 ? 0u : 1u);
+          const uint64_t vd = vdesc0 + ((vs * C::V_BYTES) >> 4);
 #pragma unroll
-          for (int kk = 1; kk < BN / 16; ++kk)
-            mma_ts(tmem + C::COL_O, sb + kk * 8, vd + ((kk * 2048) >> 4), C::IDESC_PV, 1u);
-          mma_commit(&bars.pv_done[sbi]);
-          mma_commit(&bars.vempty[vs]);
-          if (j == w.T - 1) mma_commit(&bars.o_full);
+          for (int kk = 0; kk < BN / 16; ++kk) {
+            const uint32_t acc = (kk > 0 || j > 0) ? 1u : 0u;
+            if (PAIR)
+              mma_ts_pair(tmem + C::COL_O, sb + kk * 8, vd + ((kk * 2048) >> 4), C::IDESC_PV, acc);
+            else
+              mma_ts(tmem + C::COL_O, sb + kk * 8, vd + ((kk * 2048) >> 4), C::IDESC_PV, acc);
+          }
+          if (PAIR) {
+            mma_commit_pair_both(&bars.pv_done[sbi]);
+            mma_commit_pair_both(&bars.vempty[vs]);
+            if (j == w.T - 1) mma_commit_pair_both(&bars.o_full);
+          } else {
+            mma_commit(&bars.pv_done[sbi]);
+            mma_commit(&bars.vempty[vs]);
+            if (j == w.T - 1) mma_commit(&bars.o_full);
+          }
         }
       }
       if (!ok)
         while (items.next(p, iq, &abort_sh) >= 0) {}
-      mma_commit(&bars.drain2);
+      if (PAIR)
+        mma_commit_pair_local(&bars.drain2);
+      else
+        mma_commit(&bars.drain2);
       wait_drain(&bars.drain2, 0, p.err);
     }
   } else if (warp == 11) {
@@ -475,15 +568,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           const int krow = (int)(tile_index(w, j) * BN);
-          mbar_arrive_expect_tx(&bars.vfull[s], C::KV_BYTES);
-          for (int ch = 0; ch < C::CHUNKS; ++ch)
-            tma_load_3d(vring + s * C::KV_BYTES + ch * (BN * 128), &tmV, &bars.vfull[s], ch * 64, krow, kz);
+          if (PAIR) {
+            // this CTA's half of the tile's value columns, counted on the leader's barrier
+            if (leader) mbar_arrive_expect_tx(&bars.vfull[s], 2 * C::V_BYTES);
+            tma_load_3d_pair(vring + s * C::V_BYTES, &tmV, at_leader(&bars.vfull[s]), (int)rank * (D / 2), krow, kz);
+          } else {
+            mbar_arrive_expect_tx(&bars.vfull[s], C::V_BYTES);
+            for (int ch = 0; ch < C::V_CHUNKS; ++ch)
+              tma_load_3d(vring + s * C::V_BYTES + ch * (BN * 128), &tmV, &bars.vfull[s], ch * 64, krow, kz);
+          }
           ++c;
         }
       }
       if (!ok)  // after an early exit, read the item queue to its end marker
         while (items.next(p, iq, &abort_sh) >= 0) {}
-      for (int u = (c > C::NV ? c - C::NV : 0); u < c; ++u) wait_drain(&bars.vfull[u % C::NV], (u / C::NV) & 1, p.err);
+      if (!PAIR || leader)
+        for (int u = (c > C::NV ? c - C::NV : 0); u < c; ++u)
+          wait_drain(&bars.vfull[u % C::NV], (u / C::NV) & 1, p.err);
     }
   } else if (warp < 4) {
     // ================================================================ softmax
@@ -576,7 +677,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         // P(g-1+NSB), so the parity of PV(g-1) on its buffer is unambiguous.
         if (__any_sync(kFull, rescale)) {
           const int pb = (int)((g - 1) % C::NSB);
-          if (!__all_sync(kFull, wait_bounded(&bars.pv_done[pb], (uint32_t)((g - 1) / C::NSB) & 1, &abort_sh, p.err))) {
+          if (!__all_sync(kFull,
+                          wait_bounded(&bars.pv_done[pb], (uint32_t)((g - 1) / C::NSB) & 1, &abort_sh, p.err))) {
             ok = false;
             break;
           }
@@ -604,7 +706,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tmem_st_wait();
         tc_fence_before();
-        mbar_arrive(&bars.p_full[sbi]);
+        if (PAIR) {  // one arrival per warp, on the leader's barrier
+          __syncwarp();
+          if ((t & 31) == 0) mbar_arrive_cluster(at_leader(&bars.p_full[sbi]));
+        } else {
+          mbar_arrive(&bars.p_full[sbi]);
+        }
       }
       if (!ok) continue;  // keep reading the item sequence to its end
       // Publish this item's row sum and max to the epilogue.
@@ -667,7 +774,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                            r[ch * 32 + pc * 4 + 3]);
       }
       fence_proxy_async_smem();  // the tensor core reads the rotated tile
-      mbar_arrive(&bars.qt_ready[buf]);
+      if (PAIR) {  // one arrival per warp, on the leader's barrier
+        __syncwarp();
+        if ((e & 31) == 0) mbar_arrive_cluster(at_leader(&bars.qt_ready[buf]));
+      } else {
+        mbar_arrive(&bars.qt_ready[buf]);
+      }
     };
     ItemReader<DYN, true> items{(long long)blockIdx.x};
     long long item = items.next(p, iq, &abort_sh);
@@ -689,7 +801,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       float o[D];
       tmem_ld_row<D>(tmem + la + C::COL_O, o);
       tc_fence_before();
-      mbar_arrive(&bars.o_free);
+      if (PAIR) {  // one arrival per warp, on the leader's barrier
+        __syncwarp();
+        if ((e & 31) == 0) mbar_arrive_cluster(at_leader(&bars.o_free));
+      } else {
+        mbar_arrive(&bars.o_free);
+      }
       const long long bh = (long long)w.b * p.Hq + head;
       const float inv_l = (l_row > 0.f) ? 1.f / l_row : 0.f;
 
@@ -838,8 +955,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
+  if (PAIR) {
+    // After an abort the other CTA's copies may still be landing in this
+    // CTA's shared memory or counting on its barriers: give them time.
+    if (abort_sh) {
+      const uint64_t t0 = globaltimer_ns();
+      while (globaltimer_ns() - t0 < 200000ull) __nanosleep(1000);
+    }
+    // Neither CTA frees its TMEM or exits while the pair's MMAs, copies or
+    // arrivals may still reach it.
+    cluster_sync();
+  }
   tc_fence_after();
-  if (warp == 0) tmem_dealloc(tmem, C::TMEM_COLS);
+  if (warp == 0) {
+    if (PAIR)
+      tmem_dealloc_pair(tmem, C::TMEM_COLS);
+    else
+      tmem_dealloc(tmem, C::TMEM_COLS);
+  }
 }
 
 }  // namespace da

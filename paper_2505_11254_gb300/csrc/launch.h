@@ -10,7 +10,9 @@
 namespace da {
 
 // ROWS: the instance for row-range calls (rows from Params::q_row0 > 0).
-template <int D, int MODE, int EPI, bool ROWS = false>
+// PAIR: the two-CTA sink + window kernel (d = 128, G even, whole sequences);
+// its K map has boxes of BN / 2 rows.
+template <int D, int MODE, int EPI, bool ROWS = false, bool PAIR = false>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
                         long long n_items, cudaStream_t s);
 

@@ -32,11 +32,17 @@ class ModelError(Exception):
 
 
 class Bar:
-    def __init__(self, name):
-        self.name, self.ph = name, 0
+    """An mbarrier whose phase completes after `count` arrivals (a copy's
+    completed bytes count as one arrival)."""
+
+    def __init__(self, name, count=1):
+        self.name, self.ph, self.count, self.pending = name, 0, count, 0
 
     def arrive(self):
-        self.ph += 1
+        self.pending += 1
+        if self.pending == self.count:
+            self.pending = 0
+            self.ph += 1
 
 
 def _check_wait(bar, k):
@@ -416,3 +422,261 @@ def run_decode_ring(n_chunks, stages, warps, seed):
             full[st].arrive()
         else:
             advance(name)
+
+
+def run_pair(layout, tiles, seed, mutant=None, rescale_p=0.25, max_steps=10 ** 6):
+    """The two-CTA sink + window kernel (`attn_kernel.cuh`, PAIR): CTAs 0 (the
+    leader) and 1 run the same items (two heads of one row tile).  Each CTA
+    has its own producer, V producer, softmax and epilogue; the leader's QK and
+    PV threads issue the MMAs for both, which run in one tensor pipe.  Barriers
+    the leader waits on count both CTAs: kfull / vfull (the leader's
+    expect-tx arrival plus each CTA's copy of its half), p_full and o_free (one
+    arrival per CTA, the kernel's per-warp arrivals lumped), qt_ready with
+    RoPE; q_full without RoPE counts the leader's arrival and both Q copies.
+    The commits of s_full, pv_done, vempty, o_full and q_free arrive on both
+    CTAs' barriers; kempty, l_ready and l_free stay local.  Checked besides the
+    one-CTA hazards: an MMA never reads a K or V half, a Q tile or a P that has
+    not landed in either CTA."""
+    L, rnd = layout, random.Random(seed)
+    n = len(tiles)
+    assert not L.dyn
+    cnt_pair = 1 if mutant == "pair_one_cta_arrival" else 2
+    cnt_copy = 2 if mutant == "pair_kfull_one_half" else 3
+
+    def bars(name, k, count=1):
+        return [Bar("%s%d" % (name, i), count) for i in range(k)]
+
+    lead = {
+        "kfull": bars("kfull", L.nk, cnt_copy), "vfull": bars("vfull", L.nv, 3),
+        "q_full": bars("q_full", 2, 2 if L.rope else 3), "qt_ready": bars("qt_ready", 2, cnt_pair),
+        "p_full": bars("p_full", L.nsb, cnt_pair), "o_free": Bar("o_free", cnt_pair),
+    }
+    cta = []
+    for r in range(2):
+        c = {
+            "kempty": bars("kempty.%d." % r, L.nk), "vempty": bars("vempty.%d." % r, L.nv),
+            "q_free": bars("q_free.%d." % r, 2), "s_full": bars("s_full.%d." % r, L.nsb),
+            "pv_done": bars("pv_done.%d." % r, L.nsb), "o_full": Bar("o_full.%d" % r),
+            "l_ready": bars("l_ready.%d." % r, 2, 1), "l_free": bars("l_free.%d." % r, 2, 1),
+            # with RoPE each CTA's Q lands on its own barrier (its producer's arrival + the copy)
+            "q_full": bars("q_full.%d." % r, 2, 2) if (L.rope and r == 1) else lead["q_full"],
+        }
+        cta.append(c)
+
+    pipe, copies = [], []
+    done = {"qk": set(), "pv": set(), "o_read": set(), "q_rot": set(), "l_read": set(), "k": set(), "v": set(),
+            "q": set(), "p": set()}
+    first_g = []
+    g = 0
+    for T in tiles:
+        first_g.append(g)
+        g += T
+
+    def both(name, idx=None):
+        return [c[name] if idx is None else c[name][idx] for c in cta]
+
+    def producer(r):
+        c, nq, kc = cta[r], 0, 0
+
+        def load_q(item):
+            nonlocal nq
+            qb = nq % L.nq
+            if nq >= L.nq:
+                yield (c["q_free"][qb], nq // L.nq - 1)
+                prev = nq - L.nq
+                if first_g[prev] + tiles[prev] - 1 not in done["qk"]:
+                    raise ModelError("CTA %d reloaded Q before the last QK of item %d" % (r, prev))
+            if r == 0 or L.rope:
+                c["q_full"][qb].arrive()  # the expect-tx arrival
+            copies.append((c["q_full"][qb], ("q", r, nq)))
+            nq += 1
+
+        item = 0 if n > 0 else -1
+        if item >= 0:
+            yield from load_q(item)
+        while item >= 0:
+            for j in range(tiles[item]):
+                s = kc % L.nk
+                if kc >= L.nk:
+                    yield (c["kempty"][s], kc // L.nk - 1)
+                    if (kc - L.nk) not in done["qk"]:
+                        raise ModelError("CTA %d reloaded K slot before QK(%d) completed" % (r, kc - L.nk))
+                if r == 0:
+                    lead["kfull"][s].arrive()
+                copies.append((lead["kfull"][s], ("k", r, kc)))
+                kc += 1
+            nxt = item + 1 if item + 1 < n else -1
+            if nxt >= 0:
+                yield from load_q(nxt)
+            item = nxt
+
+    def vprod(r):
+        c, vc = cta[r], 0
+        for item in range(n):
+            for j in range(tiles[item]):
+                s = vc % L.nv
+                if vc >= L.nv:
+                    yield (c["vempty"][s], vc // L.nv - 1)
+                    if (vc - L.nv) not in done["pv"]:
+                        raise ModelError("CTA %d reloaded V slot before PV(%d) completed" % (r, vc - L.nv))
+                if r == 0:
+                    lead["vfull"][s].arrive()
+                copies.append((lead["vfull"][s], ("v", r, vc)))
+                vc += 1
+
+    def qk():
+        g = 0
+        for i in range(n):
+            qb = i % L.nq
+            yield (lead["qt_ready"][qb] if L.rope else lead["q_full"][qb], i // L.nq)
+            for j in range(tiles[i]):
+                ks, sbi = g % L.nk, g % L.nsb
+                yield (lead["kfull"][ks], g // L.nk)
+                if g >= L.nsb:
+                    yield (cta[0]["pv_done"][sbi], g // L.nsb - 1)
+                pipe.append(("qk", g, i))
+                pipe.append(("commit", both("s_full", sbi)))
+                g += 1
+            pipe.append(("commit", both("q_free", qb)))
+
+    def pv():
+        g = 0
+        for i in range(n):
+            T = tiles[i]
+            for j in range(T):
+                vs, sbi = g % L.nv, g % L.nsb
+                yield (lead["p_full"][sbi], g // L.nsb)
+                yield (lead["vfull"][vs], g // L.nv)
+                if j == 0 and i >= 1:
+                    yield (lead["o_free"], i - 1)
+                pipe.append(("pv", g, i, j == 0))
+                pipe.append(("commit", both("pv_done", sbi)))
+                if mutant == "pair_vempty_leader_only":
+                    pipe.append(("commit", [cta[0]["vempty"][vs]]))
+                else:
+                    pipe.append(("commit", both("vempty", vs)))
+                if j == T - 1:
+                    pipe.append(("commit", both("o_full")))
+                g += 1
+
+    def softmax(r):
+        c, g = cta[r], 0
+        for i in range(n):
+            for j in range(tiles[i]):
+                sbi = g % L.nsb
+                yield (c["s_full"][sbi], g // L.nsb)
+                if g not in done["qk"]:
+                    raise ModelError("CTA %d softmax read S(%d) before its QK completed" % (r, g))
+                c["kempty"][g % L.nk].arrive()
+                if j >= 1 and rnd.random() < rescale_p:
+                    yield (c["pv_done"][(g - 1) % L.nsb], (g - 1) // L.nsb)
+                    if (g - 1) not in done["pv"]:
+                        raise ModelError("CTA %d rescaled O before PV(%d) completed" % (r, g - 1))
+                done["p"].add((r, g))
+                lead["p_full"][sbi].arrive()
+                yield None
+                g += 1
+            if i >= 2:
+                yield (c["l_free"][i & 1], (i >> 1) - 1)
+                if (r, i - 2) not in done["l_read"]:
+                    raise ModelError("CTA %d row sums of item %d overwritten before read" % (r, i - 2))
+            c["l_ready"][i & 1].arrive()
+
+    def epilogue(r):
+        c, nq = cta[r], 0
+
+        def rotate(buf, qi):
+            nonlocal nq
+            if L.rope:
+                yield (c["q_full"][buf], nq // L.nq)
+                if (r, qi) not in done["q"]:
+                    raise ModelError("CTA %d rotated Q of item %d before it landed" % (r, qi))
+                nq += 1
+                done["q_rot"].add((r, qi))
+                lead["qt_ready"][buf].arrive()
+
+        if n > 0:
+            yield from rotate(0, 0)
+        for i in range(n):
+            if i + 1 < n:
+                yield from rotate((i + 1) % L.nq, i + 1)
+            yield (c["l_ready"][i & 1], i >> 1)
+            done["l_read"].add((r, i))
+            c["l_free"][i & 1].arrive()
+            yield (c["o_full"], i)
+            done["o_read"].add((r, i))
+            lead["o_free"].arrive()
+
+    roles = {"qk": qk(), "pv": pv()}
+    for r in range(2):
+        roles["producer%d" % r] = producer(r)
+        roles["vprod%d" % r] = vprod(r)
+        roles["softmax%d" % r] = softmax(r)
+        roles["epilogue%d" % r] = epilogue(r)
+    waits, finished = {}, set()
+
+    def advance(name):
+        try:
+            waits[name] = next(roles[name])
+        except StopIteration:
+            finished.add(name)
+            waits[name] = None
+
+    for name in roles:
+        advance(name)
+    speed = {name: rnd.choice([0.05, 0.3, 1.0, 1.0, 3.0]) for name in list(roles) + ["pipe", "copy"]}
+    for _ in range(max_steps):
+        cands = [("role", nm) for nm in roles
+                 if nm not in finished and (waits[nm] is None or _check_wait(*waits[nm]))]
+        if pipe:
+            cands.append(("pipe", None))
+        if copies:
+            cands.append(("copy", None))
+        if not cands:
+            if len(finished) == len(roles):
+                return
+            raise ModelError("deadlock: " + "; ".join(
+                "%s waits %s for phase %d (%d completed)" % (nm, waits[nm][0].name, waits[nm][1], waits[nm][0].ph)
+                for nm in roles if nm not in finished and waits[nm] is not None))
+        kind, name = rnd.choices(cands, weights=[speed[c[1] if c[0] == "role" else c[0]] for c in cands])[0]
+        if kind == "role":
+            advance(name)
+        elif kind == "pipe":
+            op = pipe.pop(0)
+            if op[0] == "qk":
+                gg, item = op[1], op[2]
+                if gg >= L.nsb and (gg - L.nsb) not in done["pv"]:
+                    raise ModelError("QK(%d) overwrote S/P before PV(%d) read it" % (gg, gg - L.nsb))
+                for r in range(2):
+                    if ("k", r, gg) not in done["k"]:
+                        raise ModelError("QK(%d) read CTA %d's K half before it landed" % (gg, r))
+                    if (r, item) not in (done["q_rot"] if L.rope else done["q"]):
+                        raise ModelError("QK of item %d read CTA %d's Q before it was ready" % (item, r))
+                done["qk"].add(gg)
+            elif op[0] == "pv":
+                gg, item, first = op[1], op[2], op[3]
+                for r in range(2):
+                    if ("v", r, gg) not in done["v"]:
+                        raise ModelError("PV(%d) read CTA %d's V half before it landed" % (gg, r))
+                    if (r, gg) not in done["p"]:
+                        raise ModelError("PV(%d) read CTA %d's P before it was written" % (gg, r))
+                    if first and item >= 1 and (r, item - 1) not in done["o_read"]:
+                        raise ModelError("first PV of item %d overwrote CTA %d's O before it was read" % (item, r))
+                done["pv"].add(gg)
+            else:
+                for b in op[1]:
+                    b.arrive()
+        else:
+            b, what = copies.pop(rnd.randrange(len(copies)))
+            if what[0] == "q":
+                done["q"].add((what[1], what[2]))
+            else:
+                done[what[0]].add(what)
+            b.arrive()
+    raise ModelError("no end after %d steps" % max_steps)
+
+
+# Each breaks the pair protocol in one place: the leader waits for one CTA's
+# arrival instead of both (P, O, rotated Q), for one K half instead of two, or
+# the V slots are released in the leader only.
+PAIR_MUTANTS = ["pair_one_cta_arrival", "pair_kfull_one_half", "pair_vempty_leader_only"]

@@ -9,12 +9,15 @@ windows, so the ring and buffer indices wrap at every offset.  Deliberately
 broken protocols (a dropped wait each) must be caught, which shows that the
 model sees what it is meant to.  The decode kernel's K/V ring is checked the
 same way: the deployed eight- and four-stage rings over four consumer warps
-pass, a six-stage ring (stages shared between warps) must be flagged."""
+pass, a six-stage ring (stages shared between warps) must be flagged.  The
+two-CTA sink + window kernel (two heads of a row tile in a CTA pair, the
+leader issuing every MMA) is modelled with both CTAs' roles; its mutants
+drop one CTA's share of a barrier."""
 import random
 
 import pytest
 
-from pipeline_model import MUTANTS, Layout, ModelError, run, run_decode_ring
+from pipeline_model import MUTANTS, PAIR_MUTANTS, Layout, ModelError, run, run_decode_ring, run_pair
 
 LAYOUTS = {
     "sink_window_d128": Layout(dense=False, nq=1),
@@ -78,3 +81,34 @@ def test_decode_ring_with_shared_stages_is_caught():
         except ModelError:
             return
     pytest.fail("the shared-stage ring was not caught")
+
+
+PAIR_LAYOUTS = {  # deployed: two Q buffers, five K and four V slots (of half tiles)
+    "pair_sink_window_d128": Layout(dense=False, nq=2, nk=5, nv=4),
+    "pair_sink_window_d128_rope": Layout(dense=False, nq=2, nk=5, nv=4, rope=True),
+    "pair_sink_window_d128_nq1": Layout(dense=False, nq=1, nk=6, nv=5),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PAIR_LAYOUTS))
+def test_pair_protocol_holds_over_random_interleavings(name):
+    rnd = random.Random(hash(name) & 0xffff)
+    for r in range(300):
+        tiles = _items(rnd)
+        try:
+            run_pair(PAIR_LAYOUTS[name], tiles, seed=r)
+        except ModelError as e:
+            pytest.fail("%s, items %s, seed %d: %s" % (name, tiles, r, e))
+
+
+@pytest.mark.parametrize("mutant", PAIR_MUTANTS)
+def test_pair_mutant_is_caught(mutant):
+    rnd = random.Random(11)
+    for r in range(400):
+        tiles = _items(rnd) + [18, 3]
+        for lay in (PAIR_LAYOUTS["pair_sink_window_d128"], PAIR_LAYOUTS["pair_sink_window_d128_rope"]):
+            try:
+                run_pair(lay, tiles, seed=r, mutant=mutant)
+            except ModelError:
+                return
+    pytest.fail("mutant %s was not caught" % mutant)
