@@ -369,6 +369,7 @@ def time_variants(args, w, q, k, v, out, stream, restore):
                      "tail_dense_pairs_per_head": flops.tail_pairs_per_head(w.N, tail)}
         del ws
     res["rope_prefill"] = time_rope_prefill(w, q, k, v, out, stream)
+    res["standalone"] = time_standalone(w, q, k, v, stream)
     res["decode"] = time_decode(w, q, k, v, stream)
     restore()  # `out` back to the Delta result for the spot check
     return res
@@ -399,6 +400,51 @@ def time_rope_prefill(w, q, k, v, out, stream):
     ms = statistics.median(times)
     return {"ms": ms, "tokens_per_s": w.B * w.N / (ms / 1e3), "rope_base": 500000.0,
             "note": "K rotated in place (one pass), Q rotated inside the attention kernels"}
+
+
+def time_standalone(w, q, k, v, stream):
+    """The three parts through their own entry points, the unfused order of
+    Alg. 1: sparse_window_attn (bf16 S and the fp32 sparse rows at the
+    samples), strided_dense_attn (fp32 dense rows at the samples), then
+    delta_apply adding Delta_k to every row in place (one more read and write
+    of O than the fused prefill).  Median over 10 calls after 3 warm-ups, with
+    events between the three calls; delta_apply's bytes (O read and written
+    in bf16, both sampled-row sets read in fp32) against the measured HBM copy
+    bandwidth."""
+    from paper_2505_11254_gb300 import binding
+    peaks, _ = load_peaks()
+    ns = -(-w.N // w.gamma)
+    o = torch.empty_like(q)
+    s_s = torch.empty((w.B, w.Hq, ns, w.d), dtype=torch.float32, device=q.device)
+    d_s = torch.empty_like(s_s)
+    dws = binding.alloc_workspace(binding.strided_dense_workspace_size(w.B, w.Hq, w.Hkv, w.N, w.d, w.gamma),
+                                  q.device)
+
+    def call(evs):
+        evs[0].record(stream)
+        binding.sparse_window_attn(q, k, v, w.n_sink, w.window, w.gamma, out=o, s_sampled=s_s)
+        evs[1].record(stream)
+        binding.strided_dense_attn(q, k, v, w.gamma, out=d_s, workspace=dws)
+        evs[2].record(stream)
+        binding.delta_apply(o, s_s, d_s, w.gamma, out=o)
+        evs[3].record(stream)
+
+    rows = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(13)]
+    for r in rows:
+        call(r)
+    torch.cuda.synchronize()
+    if binding.check() != binding.DA_OK:
+        raise RuntimeError("device status after the standalone timing")
+    rows = rows[3:]
+    parts = {name: statistics.median(r[i].elapsed_time(r[i + 1]) for r in rows)
+             for i, name in enumerate(("sparse_window_attn", "strided_dense_attn", "delta_apply"))}
+    total = statistics.median(r[0].elapsed_time(r[3]) for r in rows)
+    apply_bytes = 2 * w.B * w.Hq * w.N * w.d * 2 + 2 * w.B * w.Hq * ns * w.d * 4
+    hbm = float(peaks.get("hbm_gbs", PEAKS_FALLBACK["hbm_gbs"]))
+    gbs = apply_bytes / (parts["delta_apply"] / 1e3) / 1e9
+    return {"ms": total, "tokens_per_s": w.B * w.N / (total / 1e3), "parts_ms": parts,
+            "delta_apply_bytes": apply_bytes, "delta_apply_gbs": gbs, "delta_apply_frac_of_hbm": gbs / hbm,
+            "note": "three entry points; the fused prefill writes O once instead"}
 
 
 def time_decode(w, q, k, v, stream):

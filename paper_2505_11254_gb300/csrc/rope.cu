@@ -31,33 +31,41 @@ __global__ void __launch_bounds__(256) rope_table_kernel(long long n_pos, int d,
   }
 }
 
-// One thread per (row, 8 pairs): channels c..c+7 and c+d/2..c+d/2+7.
+// One thread per (position, 8 pairs): channels c..c+7 and c+d/2..c+d/2+7 of
+// every row at that position.  x holds rows/N slabs of N rows (one per
+// batch and head) and slab row i is at position pos0 + i, so the thread reads
+// its 64 bytes of the table once and rotates the same channels of every slab
+// (a thread per row re-read the table once per slab: 2.3x the bytes of x at
+// 8 KV heads).
 __global__ void __launch_bounds__(256) rope_apply_kernel(__nv_bfloat16* x, long long rows, long long N, int d,
                                                          long long pos0, const float2* __restrict__ table) {
   const int h = d / 2, groups = h / 8;
-  const long long total = rows * groups;
+  const long long total = N * groups;
   for (long long t = blockIdx.x * (long long)blockDim.x + threadIdx.x; t < total;
        t += (long long)gridDim.x * blockDim.x) {
-    const long long r = t / groups;
+    const long long i = t / groups;
     const int c0 = (int)(t % groups) * 8;
-    const long long pos = pos0 + r % N;
-    __nv_bfloat16* lo = x + r * d + c0;
-    __nv_bfloat16* hi = lo + h;
-    uint4 ul = *reinterpret_cast<const uint4*>(lo);
-    uint4 uh = *reinterpret_cast<const uint4*>(hi);
-    __nv_bfloat162* pl = reinterpret_cast<__nv_bfloat162*>(&ul);
-    __nv_bfloat162* ph = reinterpret_cast<__nv_bfloat162*>(&uh);
-    const float4* tb = reinterpret_cast<const float4*>(table + pos * h + c0);
+    const float4* tb = reinterpret_cast<const float4*>(table + (pos0 + i) * h + c0);
+    float4 cs[4];  // (cos, sin) of channels c0 + 2e and c0 + 2e + 1
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float4 cs = tb[e];  // (cos, sin) of channels c0 + 2e and c0 + 2e + 1
-      const float2 a = __bfloat1622float2(pl[e]);
-      const float2 b = __bfloat1622float2(ph[e]);
-      pl[e] = __floats2bfloat162_rn(a.x * cs.x - b.x * cs.y, a.y * cs.z - b.y * cs.w);
-      ph[e] = __floats2bfloat162_rn(b.x * cs.x + a.x * cs.y, b.y * cs.z + a.y * cs.w);
+    for (int e = 0; e < 4; ++e) cs[e] = tb[e];
+    for (long long r = i; r < rows; r += N) {
+      __nv_bfloat16* lo = x + r * d + c0;
+      __nv_bfloat16* hi = lo + h;
+      uint4 ul = *reinterpret_cast<const uint4*>(lo);
+      uint4 uh = *reinterpret_cast<const uint4*>(hi);
+      __nv_bfloat162* pl = reinterpret_cast<__nv_bfloat162*>(&ul);
+      __nv_bfloat162* ph = reinterpret_cast<__nv_bfloat162*>(&uh);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float2 a = __bfloat1622float2(pl[e]);
+        const float2 b = __bfloat1622float2(ph[e]);
+        pl[e] = __floats2bfloat162_rn(a.x * cs[e].x - b.x * cs[e].y, a.y * cs[e].z - b.y * cs[e].w);
+        ph[e] = __floats2bfloat162_rn(b.x * cs[e].x + a.x * cs[e].y, b.y * cs[e].z + a.y * cs[e].w);
+      }
+      *reinterpret_cast<uint4*>(lo) = ul;
+      *reinterpret_cast<uint4*>(hi) = uh;
     }
-    *reinterpret_cast<uint4*>(lo) = ul;
-    *reinterpret_cast<uint4*>(hi) = uh;
   }
 }
 
@@ -70,7 +78,7 @@ cudaError_t launch_rope_table(long long n_pos, int d, double base, float* table,
 
 cudaError_t launch_rope_apply(void* x, long long rows, long long N, int d, long long pos0, const float* table,
                               cudaStream_t s) {
-  const long long total = rows * (d / 16);
+  const long long total = N * (d / 16);
   const long long blocks = (total + 255) / 256 < 152LL * 32 ? (total + 255) / 256 : 152LL * 32;
   rope_apply_kernel<<<(unsigned)blocks, 256, 0, s>>>(static_cast<__nv_bfloat16*>(x), rows, N, d, pos0,
                                                       reinterpret_cast<const float2*>(table));
