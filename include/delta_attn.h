@@ -33,7 +33,7 @@
  * floating-point atomics.
  *
  * Kernel choice: the sink + window pass of a whole sequence at d = 128 with
- * an even Hq / Hkv and window >= 2048 runs as a two-CTA kernel (thread-block
+ * an even Hq / Hkv and window >= 512 runs as a two-CTA kernel (thread-block
  * clusters of two, one per pair of query heads of a KV group); other shapes
  * run the one-CTA kernel.  Both give the same bits.  The environment variable
  * DELTA_ATTN_PAIR, read at each call, overrides the choice: "0" always takes

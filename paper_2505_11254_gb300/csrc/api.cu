@@ -204,20 +204,19 @@ struct Maps {
 
 // The sink + window pass of a whole sequence runs as the two-CTA kernel when
 // the query heads of each KV group pair up (G even) at d = 128 and the window
-// spans at least 16 key tiles.  Measured on GB300 against the one-CTA kernel:
-// the same time per prefill at windows 2048 and 8192 (at a higher sustained
-// clock under the power cap: it moves half the K/V bytes through each SM's
-// shared memory and from L2), 2-3 % slower at window 512, whose 6-tile items
-// pay the pair's cross-CTA item hand-off more often.  Results are
-// bit-identical.  The environment variable DELTA_ATTN_PAIR overrides the
-// choice: 0 always takes the one-CTA kernel, 1 the two-CTA one where it
-// applies.
+// spans at least 4 key tiles.  Measured on GB300 against the one-CTA kernel:
+// the same time per prefill at windows 512, 2048 and 8192, at a higher
+// sustained clock under the power cap (it moves half the K/V bytes through
+// each SM's shared memory and from L2); shorter windows were not measured.
+// Results are bit-identical.  The environment variable DELTA_ATTN_PAIR
+// overrides the choice: 0 always takes the one-CTA kernel, 1 the two-CTA one
+// where it applies.
 bool pair_sparse(int d, const Params& p) {
   if (d != 128 || p.G % 2 != 0 || p.q_row0 != 0) return false;
   const char* env = getenv("DELTA_ATTN_PAIR");
   if (env != nullptr && env[0] == '0') return false;
   if (env != nullptr && env[0] == '1') return true;
-  return p.window >= 16 * BN;
+  return p.window >= 4 * BN;
 }
 
 // Sampled rows row0 + k * gamma of every (b, head): Hp heads x R samples a box.

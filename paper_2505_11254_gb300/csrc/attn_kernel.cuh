@@ -439,7 +439,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t qdesc0 = sdesc_sw128(smem_u32(sQ), 16, 1024);
       const uint64_t kdesc0 = sdesc_sw128(smem_u32(ring), 16, 1024);
       const bool rope = p.rope != nullptr;
-      long long g = 0;
+      uint32_t g = 0;  // tiles so far: ring slots and phases (32-bit: cheap divisions by constants)
       bool ok = true;
       ItemReader<DYN, false> items{(long long)blockIdx.x};
       int i = 0;
@@ -501,7 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     regs_decrease<kRegsControl>();
     if ((tid & 31) == 0 && leader) {
       const uint64_t vdesc0 = sdesc_sw128(smem_u32(vring), BN * 128, 1024);
-      long long g = 0;
+      uint32_t g = 0;  // tiles so far: ring slots and phases (32-bit: cheap divisions by constants)
       bool ok = true;
       ItemReader<DYN, false> items{(long long)blockIdx.x};
       int i = 0;
@@ -593,7 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t la = lane_base(warp);
     const float scale = p.scale_log2;
     const uint64_t scale2 = f2_pack(scale, scale);
-    long long g = 0;
+    uint32_t g = 0;  // tiles so far (32-bit: cheap divisions by constants)
     bool ok = true;
     int i = 0;
     ItemReader<DYN, true> items{(long long)blockIdx.x};

@@ -2,7 +2,7 @@
 a time, one MMA issuer for both CTAs of a cluster) against the fp64 oracle and
 against the one-CTA kernel, through the C ABI (DELTA_ATTN_PAIR=1 / 0 select
 them).  The library takes the two-CTA kernel for whole sequences at d = 128
-with an even GQA ratio and a window of at least 2048 keys; the tests force it
+with an even GQA ratio and a window of at least 512 keys; the tests force it
 at every window, and the cases cover every epilogue it is built with (the Delta
 fused in the row tile, the separate Delta pass, bf16 rows for the recompute
 form and sparse_window_attn, the smoothed correction), the RoPE rotation of Q
@@ -169,11 +169,11 @@ def test_pair_repeated_calls_bit_identical():
 
 def test_default_choice_follows_the_window():
     """Without the override the two kernels give the same bits at a short and a
-    long window (the library picks one-CTA at window 512 and two-CTA at 2048)."""
+    long window (the library picks one-CTA at window 256 and two-CTA at 2048)."""
     q, k, v = rand_qkv(1, 4, 2, 4608, 128, seed=12)
     env = os.environ.pop("DELTA_ATTN_PAIR")
     try:
-        for w in (512, 2048):
+        for w in (256, 2048):
             a = binding.delta_attn_prefill(q, k, v, 4, w, 64)
             with one_cta_kernel():
                 b = binding.delta_attn_prefill(q, k, v, 4, w, 64)
