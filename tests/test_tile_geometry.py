@@ -3,7 +3,8 @@ with g++): the per-item range of tiles that skip the element-wise mask agrees
 with the per-tile predicate, no skipped tile holds an invisible (row, key)
 pair, the split-K units cover each dense M-tile once, and every lane maps to
 its query head's KV head with each (batch, head, row) held once, over many
-shapes, all three modes, the dense tail and the GQA head packings."""
+shapes, all three modes, the dense tail and the GQA head packings; and the
+two-CTA kernel's clusters always pair two heads of one row tile."""
 import os
 import shutil
 import subprocess

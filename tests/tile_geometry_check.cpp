@@ -8,7 +8,9 @@
 // library's planner (plan.h) lays them out, cover every M-tile's causal key
 // range exactly once with the partial slots and tickets the merge assumes.  For every head packing of the dense tiles (GQA 1, 2,
 // 3, 4 and 16), each lane's query head reads its own KV head (floor(h / G))
-// and every (batch, head, row or sample) sits in exactly one lane.
+// and every (batch, head, row or sample) sits in exactly one lane.  For the
+// two-CTA sink + window kernel, the items the two CTAs of a cluster take
+// together are two heads of one row tile with the same key tiles.
 #define __host__
 #define __device__
 #define __forceinline__ inline
@@ -210,6 +212,43 @@ static const PlanCase kPlans[] = {{152, {kMaxLevelsUsed, kUnitTiles, kMinChunk, 
                                   {152, {kMaxLevelsUsed, 3, 1, 0}},
                                   {1, {kMaxLevels, 1, 1, kLevelPartialBytes}}};
 
+// The two-CTA sink + window kernel (G even, whole sequences): the CTAs 2c and
+// 2c + 1 of a cluster walk items 2c + k grid and 2c + 1 + k grid.  With G and
+// the grid even these are always the two heads h0, h0 + 1 of one KV group and
+// one row tile, whose key-tile lists and masked-tile ranges are identical, and
+// both CTAs see the same number of items: the leader's MMAs serve both.
+static int check_pairs(const Params& p) {
+  int bad = 0;
+  const long long n = (long long)p.B * p.Hq * p.qtiles;
+  if (n % 2 != 0) {
+    std::printf("pairs: odd item count %lld\n", n);
+    return 1;
+  }
+  for (long long lin = 0; lin < n; lin += 2) {
+    const Work a = decode_work<MODE_SPARSE>(p, lin), b = decode_work<MODE_SPARSE>(p, lin + 1);
+    bool same = a.b == b.b && a.g == b.g && b.h0 == a.h0 + 1 && a.r0 == b.r0 && a.r_last == b.r_last &&
+                a.kt_lo == b.kt_lo && a.kt_hi == b.kt_hi && a.n_sink_tiles == b.n_sink_tiles && a.T == b.T;
+    int a0, a1, b0, b1;
+    unmasked_tiles<MODE_SPARSE>(p, a, a0, a1);
+    unmasked_tiles<MODE_SPARSE>(p, b, b0, b1);
+    same = same && a0 == b0 && a1 == b1;
+    for (int j = 0; same && j < a.T; ++j) same = tile_index(a, j) == tile_index(b, j);
+    if (!same) {
+      if (bad < 5) std::printf("pairs: items %lld and %lld differ (heads %d, %d)\n", lin, lin + 1, a.h0, b.h0);
+      ++bad;
+    }
+  }
+  for (long long grid : {2LL, 148LL, 150LL, 152LL}) {
+    for (long long c = 0; 2 * c < grid; ++c)
+      for (long long x = 2 * c; x < n || x + 1 < n; x += grid)
+        if ((x < n) != (x + 1 < n)) {
+          if (bad < 5) std::printf("pairs: grid %lld cluster %lld sees unequal item counts\n", grid, c);
+          ++bad;
+        }
+  }
+  return bad;
+}
+
 // q_row0: a row-range call computing rows [q_row0, N) (0: the whole sequence).
 static int check_shape(int B, int Hq, int Hkv, long long N, long long win, int ns, int gm, long long q_row0 = 0) {
   int bad = 0;
@@ -222,6 +261,7 @@ static int check_shape(int B, int Hq, int Hkv, long long N, long long win, int n
   p.qtiles = (N - q_row0 + BM - 1) / BM;
   plan_split_k(p, 152, 128);
   bad += check<MODE_SPARSE>(p, (long long)p.B * p.Hq * p.qtiles);
+  if (q_row0 == 0 && p.G % 2 == 0) bad += check_pairs(p);
   bad += check<MODE_STRIDED_SPARSE>(p, (long long)p.B * p.groups_per_b * p.mtiles);
   {  // the library's own policy for this shape
     Params q = p;
