@@ -1,9 +1,13 @@
 // launch_impl.cuh — the launcher template; included by the attn_*.cu units.
 #pragma once
+#include <atomic>
+
 #include "attn_kernel.cuh"
 #include "launch.h"
 
 namespace da {
+
+constexpr int kMaxDevices = 64;
 
 // Persistent launch: min(items, SMs) CTAs, each walking items with a stride
 // of the grid size.  The two-CTA kernel runs in clusters of two, as many as
@@ -39,8 +43,14 @@ cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUte
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cfg.gridDim = dim3((unsigned)(2 * (sms / 2)));
-  int clusters = 0;
-  if ((e = cudaOccupancyMaxActiveClusters(&clusters, kfn, &cfg)) != cudaSuccess) return e;
+  // Clusters that fit at once: a property of the device and this instance,
+  // asked once per device (racing first calls compute the same value).
+  static std::atomic<int> fit[kMaxDevices];
+  int clusters = dev < kMaxDevices ? fit[dev].load(std::memory_order_relaxed) : 0;
+  if (clusters == 0) {
+    if ((e = cudaOccupancyMaxActiveClusters(&clusters, kfn, &cfg)) != cudaSuccess) return e;
+    if (dev < kMaxDevices) fit[dev].store(clusters, std::memory_order_relaxed);
+  }
   if (clusters < 1) return cudaErrorInvalidConfiguration;
   long long grid = 2LL * clusters;
   if (grid > n_items) grid = n_items;
