@@ -97,6 +97,7 @@ struct Cfg {
   // warpgroup, or in a pair one per warp of both CTAs.
   static constexpr uint32_t ARRIVALS = PAIR ? 8 : 128;
   static_assert(COL_O + D <= TMEM_COLS, "TMEM layout");
+  static_assert(BN == 128, "the softmax loads S in two 64-column halves and stores P in two 32-column halves");
   static_assert(NK <= 8 && NV <= 8, "ring barriers");
   static_assert(SMEM <= 232448, "shared memory above the 227 KB per-block limit");
 };
@@ -616,7 +617,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const uint32_t sb = C::COL_S + (uint32_t)sbi * BN;
         float s[BN];
-        tmem_ld_row<BN>(tmem + la + sb, s);
+        {  // S(g): two 64-column loads (fewer, wider TMEM loads than 32-column ones measured faster)
+          uint32_t r0[64], r1[64];
+          tmem_ld64(tmem + la + sb, r0);
+          tmem_ld64(tmem + la + sb + 64, r1);
+          tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 64; ++c) {
+            s[c] = __uint_as_float(r0[c]);
+            s[c + 64] = __uint_as_float(r1[c]);
+          }
+        }
         if (j < j_plain0 || j >= j_plain1) {
           // Visible key offsets c of this tile: lo <= c <= hi (window and
           // causality), plus c < se (sinks), turned into one 32-bit word of
@@ -698,11 +709,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         l_run += l_tile;
         m_run = m_use;
 #pragma unroll
-        for (int q = 0; q < BN / 32; ++q) {
-          uint32_t r[16];
+        for (int q = 0; q < BN / 64; ++q) {
+          uint32_t r[32];
 #pragma unroll
-          for (int c = 0; c < 16; ++c) r[c] = pk[q * 16 + c];
-          tmem_st16(tmem + la + sb + q * 16, r);
+          for (int c = 0; c < 32; ++c) r[c] = pk[q * 32 + c];
+          tmem_st32(tmem + la + sb + q * 32, r);
         }
         tmem_st_wait();
         tc_fence_before();
