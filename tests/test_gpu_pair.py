@@ -80,6 +80,8 @@ CASES = [
     (1, 8, 2, 8192, 128, 4, 512, 64),     # 512 items: several per CTA, rings wrap
     (1, 4, 2, 1200, 128, 17, 200, 16),    # 17 sinks: a full-width sink tile
     (1, 4, 2, 700, 128, 4, 2048, 32),     # window >= N: every row dense
+    (1, 2, 1, 1, 128, 4, 512, 4),         # N = 1: two items, one cluster
+    (1, 4, 2, 130, 128, 0, 512, 2),       # no sinks, a 2-row ragged tile, gamma 2
 ]
 
 
