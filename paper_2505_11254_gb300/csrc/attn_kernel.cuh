@@ -34,6 +34,10 @@
 // the device status word, the roles stop working (keeping every named barrier
 // and warp-collective instruction uniform), drain their in-flight copies and
 // MMAs, free TMEM and return.
+// The sink + window pass also comes as a two-CTA form (PAIR, see Cfg): a
+// cluster of two CTAs takes two query heads of one row tile, the leader's
+// warps 9 and 10 issue cta_group::2 MMAs for both, and each CTA holds half of
+// every K and V tile.
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
