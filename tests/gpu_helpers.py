@@ -38,3 +38,28 @@ def assert_close(got, ref, what, max_abs=MAX_ABS, mean_abs=MEAN_ABS):
     mx, mn = float(err.max()) if err.size else 0.0, float(err.mean()) if err.size else 0.0
     assert mx <= max_abs and mn <= mean_abs, "%s: max-abs %.3g mean-abs %.3g" % (what, mx, mn)
     return mx, mn
+
+
+GUARD = 4096   # guard bytes on each side
+PATTERN = 0xA5
+
+
+class Guarded:
+    """A tensor of the given shape and dtype inside a buffer with guard bytes
+    on both sides, 256-byte aligned like a fresh allocation."""
+
+    def __init__(self, shape, dtype, device="cuda"):
+        self.nbytes = int(torch.tensor([], dtype=dtype).element_size() * torch.Size(shape).numel())
+        self.buf = torch.full((2 * GUARD + self.nbytes + 256,), PATTERN, dtype=torch.uint8, device=device)
+        self.t = self.buf[GUARD:GUARD + self.nbytes].view(dtype).view(shape)
+
+    def intact(self):
+        if self.buf.is_cuda:
+            torch.cuda.synchronize()
+        head = self.buf[:GUARD]
+        tail = self.buf[GUARD + self.nbytes:]
+        return bool((head == PATTERN).all()) and bool((tail == PATTERN).all())
+
+
+def guarded_ws(nbytes, device="cuda"):
+    return Guarded((max(int(nbytes), 16),), torch.uint8, device)
