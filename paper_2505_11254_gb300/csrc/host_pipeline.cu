@@ -19,6 +19,8 @@
 #include <mutex>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "delta_attn.h"
 
 namespace {
@@ -95,6 +97,10 @@ int delta_attn_host_workspace_size(int B, int Hq, int Hkv, int64_t N, int d, int
 int delta_attn_prefill_host(const void* Qh, const void* Kh, const void* Vh, void* Oh, int B, int Hq, int Hkv,
                             int64_t N, int d, int n_sink, int64_t window, int gamma, void* workspace,
                             size_t ws_bytes, void* stream) {
+  nvtxRangePushA("delta_attn_prefill_host");
+  struct Pop {
+    ~Pop() { nvtxRangePop(); }
+  } nvtx_pop;
   if (!Qh || !Kh || !Vh || !Oh) return DA_ERR_INVALID_ARG;
   HostPlan hp;
   int rc = make_host_plan(B, Hq, Hkv, N, d, n_sink, window, gamma, &hp);
