@@ -268,7 +268,10 @@ cudaError_t launch(int d, const CUtensorMap& q, const CUtensorMap& k, const CUte
 // one-CTA whole-sequence kernel otherwise.
 template <int EPI>
 cudaError_t launch_sparse(int d, const Maps& m, const Params& p, long long grid, cudaStream_t s) {
-  if (pair_sparse(d, p)) return launch_attn<128, MODE_SPARSE, EPI, false, true>(m.q, m.kh, m.v, p, grid, s);
+  if (pair_sparse(d, p)) {
+    const cudaError_t e = launch_attn<128, MODE_SPARSE, EPI, false, true>(m.q, m.kh, m.v, p, grid, s);
+    if (e != cudaErrorNotSupported) return e;  // else no cluster of two fits: the one-CTA kernel below
+  }
   if (p.q_row0 == 0) return launch<MODE_SPARSE, EPI>(d, m.q, m.k, m.v, p, grid, s);
   // Row ranges are Eq. 6 prefills only (delta_attn_prefill_rows).
   if constexpr (EPI == EPI_FUSED_INTILE || EPI == EPI_FUSED_DELTA) {

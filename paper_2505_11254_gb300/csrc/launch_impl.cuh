@@ -11,7 +11,8 @@ constexpr int kMaxDevices = 64;
 
 // Persistent launch: min(items, SMs) CTAs, each walking items with a stride
 // of the grid size.  The two-CTA kernel runs in clusters of two, as many as
-// fit at once (a cluster's CTAs share a GPC), and an even grid.
+// fit at once (a cluster's CTAs share a GPC), and an even grid; it returns
+// cudaErrorNotSupported, launching nothing, where no cluster of two fits.
 template <int D, int MODE, int EPI, bool ROWS, bool PAIR>
 cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv, const Params& p,
                         long long n_items, cudaStream_t s) {
@@ -44,14 +45,16 @@ cudaError_t launch_attn(const CUtensorMap& tq, const CUtensorMap& tk, const CUte
   cfg.numAttrs = 1;
   cfg.gridDim = dim3((unsigned)(2 * (sms / 2)));
   // Clusters that fit at once: a property of the device and this instance,
-  // asked once per device (racing first calls compute the same value).
+  // asked once per device (racing first calls compute the same value; -1:
+  // none fit).  When none fit the caller takes the one-CTA kernel.
   static std::atomic<int> fit[kMaxDevices];
   int clusters = dev < kMaxDevices ? fit[dev].load(std::memory_order_relaxed) : 0;
   if (clusters == 0) {
     if ((e = cudaOccupancyMaxActiveClusters(&clusters, kfn, &cfg)) != cudaSuccess) return e;
+    if (clusters < 1) clusters = -1;
     if (dev < kMaxDevices) fit[dev].store(clusters, std::memory_order_relaxed);
   }
-  if (clusters < 1) return cudaErrorInvalidConfiguration;
+  if (clusters < 1) return cudaErrorNotSupported;
   long long grid = 2LL * clusters;
   if (grid > n_items) grid = n_items;
   cfg.gridDim = dim3((unsigned)grid);
